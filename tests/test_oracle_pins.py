@@ -1,0 +1,343 @@
+"""Pins of the CPU oracle against things other than itself.
+
+Each test checks the oracle against what the paper and the mathematics fix:
+hand-derived values (tests/golden, each citing its equation), the exact
+identity between explicit deletion and Eq. 6, a textbook special case
+(uniform attention), invariants, and an independent pure-Python brute force
+over every page subset.  No GPU is needed.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import brute, core
+from paper_2608_07855_gb300 import synth
+
+INF = math.inf
+
+
+def _val(s):
+    return float(eval(str(s), {"sqrt": math.sqrt, "inf": INF}))
+
+
+def _close(a, b, rel=1e-12, abs_=1e-14):
+    if math.isinf(b) or math.isinf(a):
+        return a == b
+    return abs(a - b) <= rel * abs(b) + abs_
+
+
+def _prob_from_case(c, layer_mask=None):
+    K = np.asarray(c["K"], float)
+    V = np.asarray(c["V"], float)
+    Q = np.asarray(c["Q"], float)
+    pages = c["pages"]
+    return core.Problem(K, V, c["pos"], Q, c["qpos"], [p[0] for p in pages], [p[1] for p in pages],
+                        layer_mask=layer_mask, scale=c.get("scale"))
+
+
+@pytest.fixture(scope="module")
+def hand_cases(golden_dir):
+    with open(os.path.join(golden_dir, "effects_hand.json")) as f:
+        return json.load(f)["cases"]
+
+
+@pytest.mark.parametrize("mode", ["explicit", "closed"])
+def test_hand_effects(hand_cases, mode):
+    for c in hand_cases:
+        pb = _prob_from_case(c)
+        R, R_head = core.page_effects(pb, mode)
+        for E, want in enumerate(c["R"]):
+            assert _close(R[E], _val(want)), (c["name"], E, R[E], want)
+        if "R_head" in c:
+            for l, heads in enumerate(c["R_head"]):
+                for h, row in enumerate(heads):
+                    for E, want in enumerate(row):
+                        assert _close(R_head[l, h, E], _val(want)), (c["name"], l, h, E)
+
+
+def test_hand_sets_and_greedy(hand_cases):
+    for c in hand_cases:
+        pb = _prob_from_case(c)
+        for s in c.get("sets", []):
+            R, _ = core.set_effect(pb, s["pages"])
+            assert _close(R, _val(s["R"])), (c["name"], s)
+        for g in c.get("greedy", []):
+            for mode in ("explicit", "closed"):
+                acc, step = core.greedy(pb, g["cand"], g["tau"], mode)
+                assert sorted(np.flatnonzero(acc).tolist()) == sorted(g["accepted"]), (c["name"], g, mode)
+                for got, want in zip(step, g["step_R"]):
+                    assert _close(got, _val(want)), (c["name"], g, mode, step)
+
+
+# ----------------------------------------------------------------------------
+# random problems
+
+
+def _random_problem(rng, M=2, H=2, g=2, d=5, S=30, W=4, P=6, gapped=True, layer_mask=None,
+                    scale=None, v_scale=1.0):
+    Hq = H * g
+    K = rng.standard_normal((M, H, S, d)) * 1.5
+    V = rng.standard_normal((M, H, S, d)) * v_scale
+    Q = rng.standard_normal((M, Hq, W, d))
+    if gapped:
+        pos = np.cumsum(rng.integers(1, 4, size=S)).astype(np.int32)
+    else:
+        pos = np.arange(S, dtype=np.int32)
+    # queries at the tail, some before the last resident tokens (causal mask bites)
+    qpos = np.sort(rng.choice(pos[S // 2:], size=W, replace=False)).astype(np.int32)
+    # P pages: disjoint spans, random lengths, gaps allowed
+    cuts = np.sort(rng.choice(np.arange(1, S), size=2 * P, replace=False))
+    ps = cuts[0::2].astype(np.int32)
+    pl = np.maximum(1, np.minimum(cuts[1::2] - cuts[0::2], 6)).astype(np.int32)
+    return core.Problem(K, V, pos, Q, qpos, ps, pl, layer_mask=layer_mask, scale=scale)
+
+
+def _to_brute(pb):
+    return {"K": pb.K.tolist(), "V": pb.V.tolist(), "Q": pb.Q.tolist(), "pos": pb.pos.tolist(),
+            "qpos": pb.qpos.tolist(), "scale": pb.scale,
+            "pages": list(zip(pb.page_start.tolist(), pb.page_len.tolist()))}
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_brute_force_all_subsets(seed):
+    rng = np.random.default_rng(100 + seed)
+    mask = np.array([1, 0, 1], np.uint8) if seed % 2 else None
+    pb = _random_problem(rng, M=3, H=2, g=2, d=3, S=14, W=3, P=4, layer_mask=mask)
+    bp = _to_brute(pb)
+    layers = None if mask is None else mask.tolist()
+    table = brute.all_subset_effects(bp, layers)
+    for A, want in table.items():
+        got, _ = core.set_effect(pb, sorted(A))
+        assert _close(got, want, 1e-11), (A, got, want)
+    for mode in ("explicit", "closed"):
+        R, _ = core.page_effects(pb, mode)
+        for E in range(pb.P):
+            assert _close(R[E], table[frozenset([E])], 1e-11), (mode, E)
+    finite = sorted(set(round(v, 9) for v in table.values() if np.isfinite(v) and v > 0))
+    for trial in range(3):
+        cand = rng.permutation(pb.P).tolist()
+        k = len(finite) * (trial + 1) // 4
+        # a threshold between two attained values: no decision sits on a tie
+        tau = 0.5 * (finite[k] + finite[k + 1]) if k + 1 < len(finite) else 0.1
+        D, steps = brute.greedy_from_table(table, cand, tau)
+        for mode in ("explicit", "closed"):
+            acc, step = core.greedy(pb, cand, tau, mode)
+            assert set(np.flatnonzero(acc).tolist()) == set(D), (mode, cand, tau)
+            for a, b in zip(step, steps):
+                assert _close(a, b, 1e-11), (mode, step, steps)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_explicit_equals_closed_form(seed):
+    """Eq. 6 is an exact identity: deleting E and renormalising equals the
+    closed form built from the one unmasked softmax."""
+    rng = np.random.default_rng(seed)
+    pb = _random_problem(rng, M=2, H=2, g=3, d=16, S=200, W=6, P=25)
+    Re, He = core.page_effects(pb, "explicit")
+    Rc, Hc = core.page_effects(pb, "closed")
+    fin = np.isfinite(He)
+    assert np.array_equal(fin, np.isfinite(Hc))
+    assert np.allclose(He[fin], Hc[fin], rtol=1e-10, atol=1e-13)
+    assert (Re > 0).sum() > pb.P // 2
+
+
+def test_uniform_attention_textbook():
+    """K = 0: every visible token gets weight 1/n, so o is the plain mean of
+    the visible values and o^{\\E} the mean of the visible values outside E."""
+    rng = np.random.default_rng(7)
+    pb = _random_problem(rng, M=1, H=1, g=2, d=6, S=40, W=5, P=8)
+    K0 = np.zeros_like(pb.K)
+    pb0 = core.Problem(K0, pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len)
+    _, R_head = core.page_effects(pb0, "explicit")
+    for h in range(pb0.Hq):
+        for E in range(pb0.P):
+            want = 0.0
+            for w in range(pb0.W):
+                vis = pb0.pos <= pb0.qpos[w]
+                inE = np.zeros(pb0.S, bool)
+                inE[pb0.page_start[E]: pb0.page_start[E] + pb0.page_len[E]] = True
+                if not (vis & inE).any():
+                    r = 0.0
+                elif not (vis & ~inE).any():
+                    r = INF
+                else:
+                    o = pb0.V[0, 0, vis].mean(axis=0)
+                    o2 = pb0.V[0, 0, vis & ~inE].mean(axis=0)
+                    r = np.linalg.norm(o - o2) / np.linalg.norm(o)
+                want = max(want, r)
+            assert _close(R_head[0, h, E], want, 1e-12), (h, E)
+
+
+def test_invariants():
+    rng = np.random.default_rng(11)
+    pb = _random_problem(rng, M=2, H=2, g=2, d=8, S=60, W=5, P=10)
+    R, R_head = core.page_effects(pb, "explicit")
+    # deleting the empty set changes nothing
+    assert core.set_effect(pb, [])[0] == 0.0
+    # deleting every token visible to some query: infinite effect
+    allp = core.Problem(pb.K, pb.V, pb.pos, pb.Q, pb.qpos, [0], [pb.S])
+    assert core.page_effects(allp, "explicit")[0][0] == INF
+    # V -> cV leaves the relative effect unchanged (c != 0)
+    for c in (-2.5, 3.0):
+        pbc = core.Problem(pb.K, c * pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len)
+        assert np.allclose(core.page_effects(pbc, "explicit")[0], R, rtol=1e-11)
+    # K -> cK with scale -> scale / c leaves the scores unchanged
+    pbk = core.Problem(2.0 * pb.K, pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len,
+                       scale=pb.scale / 2.0)
+    assert np.allclose(core.page_effects(pbk, "explicit")[0], R, rtol=1e-11)
+    # GQA equals MHA with the KV heads replicated g times
+    g = pb.Hq // pb.H
+    Kr = np.repeat(pb.K, g, axis=1)
+    Vr = np.repeat(pb.V, g, axis=1)
+    pbm = core.Problem(Kr, Vr, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len)
+    assert np.allclose(core.page_effects(pbm, "explicit")[1], R_head, rtol=1e-12)
+    # layer mask: the max runs over the selected layers only
+    pbl = core.Problem(pb.K, pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len,
+                       layer_mask=np.array([0, 1], np.uint8))
+    Rl, Hl = core.page_effects(pbl, "explicit")
+    assert np.allclose(Rl, R_head[1].max(axis=0)) and (Hl[0] == 0).all()
+    # permuting the resident tokens (with their positions) leaves a set effect unchanged
+    perm = rng.permutation(pb.S)
+    A = [1, 4, 7]
+    toks = np.concatenate([np.arange(pb.page_start[E], pb.page_start[E] + pb.page_len[E]) for E in A])
+    inv = np.argsort(perm)
+    pbp = core.Problem(pb.K[:, :, perm], pb.V[:, :, perm], pb.pos[perm], pb.Q, pb.qpos,
+                       np.sort(inv[toks]), np.ones(len(toks), np.int32))
+    Rp, _ = core.set_effect(pbp, range(len(toks)))
+    assert _close(Rp, core.set_effect(pb, A)[0], 1e-11)
+
+
+def test_additive_partials_equal_joint_deletion():
+    """Eq. 11 deletes a page set at once; the closed-form greedy adds the
+    page sums of Eq. 6 instead.  Both must agree step by step."""
+    rng = np.random.default_rng(3)
+    pb = _random_problem(rng, M=2, H=2, g=2, d=8, S=120, W=5, P=14)
+    cand = rng.permutation(pb.P)[:10]
+    for tau in (0.05, 0.3, 1.0):
+        a1, s1 = core.greedy(pb, cand, tau, "explicit")
+        a2, s2 = core.greedy(pb, cand, tau, "closed")
+        assert np.array_equal(a1, a2)
+        fin = np.isfinite(s1)
+        assert np.array_equal(fin, np.isfinite(s2))
+        assert np.allclose(s1[fin], s2[fin], rtol=1e-10)
+
+
+# ----------------------------------------------------------------------------
+# classification, selection, gather
+
+
+def test_classify_hand(golden_dir):
+    with open(os.path.join(golden_dir, "classify_hand.json")) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        st, cand = core.classify(c["R_pre"], c["R_post"], c["eligible"], **c["thresholds"])
+        assert st.tolist() == c["state"], c["name"]
+        assert cand.tolist() == c["cand"], c["name"]
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_classify_properties(seed):
+    rng = np.random.default_rng(seed)
+    P = 200
+    Rm = rng.choice([0.0, 0.005, 0.01, 0.03, 0.05, 0.2], size=P) * rng.uniform(0.5, 1.5, size=P) ** (seed % 2)
+    Rp = rng.choice([0.0, 0.005, 0.01, 0.03, 0.05, 0.2], size=P)
+    el = (rng.uniform(size=P) < 0.8).astype(np.uint8)
+    st, cand = core.classify(Rm, Rp, el)
+    assert (st[el == 0] == 0).all() and (st[el == 1] > 0).all()
+    idx = np.flatnonzero(el)
+    Pm = core.percentile_ranks(Rm, idx)
+    Pp = core.percentile_ranks(Rp, idx)
+    Hm = (Rm[idx] >= np.float32(0.05)) & (Pm >= 0.75)
+    Lm = (Rm[idx] <= np.float32(0.01)) & (Pm <= 0.25)
+    assert not (Hm & Lm).any()
+    assert set(cand.tolist()) == set(np.flatnonzero(st == oracle.STATE_CANDIDATE).tolist())
+    keys = [(Rp[E], -Rm[E], E) for E in cand]
+    assert keys == sorted(keys)
+
+
+def test_select_hand(golden_dir):
+    with open(os.path.join(golden_dir, "select_hand.json")) as f:
+        g = json.load(f)
+    ps = [p[0] for p in g["pages"]]
+    pl = [p[1] for p in g["pages"]]
+    for c in g["cases"]:
+        cps = [p[0] for p in c["pages"]] if "pages" in c else ps
+        cpl = [p[1] for p in c["pages"]] if "pages" in c else pl
+        I = core.select_indices(c.get("S", g["S"]), cps, cpl, c["retired"], c["pending"],
+                                c["priority"], c.get("fill_score", g["fill_score"]), c["B"], c["B_N"],
+                                c["cap"])
+        assert I.tolist() == c["I"], c["name"]
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_select_properties(seed):
+    rng = np.random.default_rng(seed)
+    S = 400
+    cuts = np.sort(rng.choice(np.arange(1, S), size=60, replace=False))
+    ps, pl = cuts[0::2], np.minimum(cuts[1::2] - cuts[0::2], 16)
+    P = len(ps)
+    retired = (rng.uniform(size=P) < 0.3).astype(np.uint8)
+    pending = rng.choice(P, size=8, replace=False)
+    prio = rng.choice([0.1, 0.2, 0.5], size=8)
+    score = rng.choice(np.linspace(0, 1, 7), size=S).astype(np.float32)
+    B = int(rng.integers(0, 300))
+    B_N = int(B * 0.25)
+    I = core.select_indices(S, ps, pl, retired, pending, prio, score, B, B_N, 4)
+    assert len(I) <= B and (np.diff(I) > 0).all()
+    tok_ret = np.zeros(S, bool)
+    for E in np.flatnonzero(retired):
+        tok_ret[ps[E]: ps[E] + pl[E]] = True
+    assert not tok_ret[I].any()
+    N = core.protect_pending(ps, pl, retired, pending, prio, B_N, 4)
+    prot = np.concatenate([np.arange(ps[E], ps[E] + pl[E]) for E in N]) if N else np.zeros(0, int)
+    assert np.isin(prot, I).all() and len(prot) <= B_N and len(N) <= 4
+    # an independent formulation of the fill: lexicographic sort of the keys
+    rest = np.flatnonzero(~tok_ret & ~np.isin(np.arange(S), prot))
+    room = B - len(prot)
+    order = np.lexsort((-rest, -score[rest].astype(np.float64)))
+    want = np.union1d(prot, rest[order[:room]] if len(rest) > room else rest)
+    assert np.array_equal(I, want)
+
+
+def test_gather_is_indexing():
+    rng = np.random.default_rng(0)
+    K = rng.standard_normal((2, 3, 10, 4))
+    V = rng.standard_normal((2, 3, 10, 4))
+    pos = np.arange(100, 110)
+    I = np.array([0, 3, 4, 9])
+    k, v, p = core.gather(K, V, pos, I)
+    for l, h, j, c in itertools.product(range(2), range(3), range(4), range(4)):
+        assert k[l, h, j, c] == K[l, h, I[j], c] and v[l, h, j, c] == V[l, h, I[j], c]
+    assert p.tolist() == [100, 103, 104, 109]
+
+
+# ----------------------------------------------------------------------------
+
+
+def test_tiny_workload_selfcheck():
+    """The Tiny workload must give the later stages something to decide:
+    completion candidates for every seed, and a joint rejection for seed 0."""
+    cfg = synth.CONFIGS["tiny"]
+    rejections = {}
+    for seed in range(5):
+        tr = synth.make_trajectory(cfg, seed)
+        K = synth.values_f64(tr.K, cfg.dtype)
+        V = synth.values_f64(tr.V, cfg.dtype)
+        pre = core.Problem(K[:, :, :tr.L_pre], V[:, :, :tr.L_pre], tr.pos[:tr.L_pre],
+                           synth.values_f64(tr.Q_pre, cfg.dtype), tr.qpos_pre,
+                           tr.page_start[:tr.P_pre], tr.page_len[:tr.P_pre])
+        post = core.Problem(K, V, tr.pos, synth.values_f64(tr.Q_post, cfg.dtype), tr.qpos_post,
+                            tr.page_start, tr.page_len)
+        Rm = np.zeros(tr.P_post)
+        Rm[:tr.P_pre] = core.page_effects(pre, "closed")[0]
+        Rp = core.page_effects(post, "closed")[0]
+        st, cand = core.classify(Rm, Rp, tr.eligible)
+        assert len(cand) >= 1, seed
+        acc, _ = core.greedy(post, cand, cfg.tau_joint, "closed")
+        rejections[seed] = len(cand) - int(acc.sum())
+    assert rejections[0] >= 1, rejections
