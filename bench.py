@@ -1,0 +1,393 @@
+#!/usr/bin/env python3
+"""CommitKV hot-path benchmark on GB300.
+
+A step is one pass of the whole hot path over one synthetic agent-shaped
+trajectory batch: pre-commit scoring, post-commit scoring, classification,
+greedy joint test and the compaction checkpoint (five C-ABI calls on one
+stream).  The metric is KV tokens scored per second, (L_pre + L_post) per
+trajectory per step, over whole steps, with inputs resident in HBM.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
+                    [--impl ours|reference]
+
+N > 1 runs under torchrun: every rank scores its own trajectories (no
+data-path collective; weak scaling), the timing is a barrier plus the max
+over ranks.  --impl reference times the CPU oracle (the only reference for
+a paper without code) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="qwen3_8b_32k")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.flush()
+        self.f.seek(0)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.f.read().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.f.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------
+# CPU baseline: the oracle, as it stands, on a bounded sample
+
+
+def oracle_sample(cfg, tr, budget_s: float):
+    """Time the oracle's closed-form page effects (pre + post) on the first
+    layers of the workload until about budget_s seconds of CPU work.
+    Returns (tokens scored per second extrapolated to the whole workload,
+    threads used, description)."""
+    import oracle
+    from paper_2608_07855_gb300 import synth
+
+    L = tr.L_pre
+    done_layers, elapsed = 0, 0.0
+    threads = min(os.cpu_count() or 1, cfg.Hq)
+    while done_layers < cfg.M and elapsed < budget_s:
+        l = done_layers
+        K = synth.values_f64(tr.K[l:l + 1], cfg.dtype)
+        V = synth.values_f64(tr.V[l:l + 1], cfg.dtype)
+        pre = oracle.Problem(K[:, :, :L], V[:, :, :L], tr.pos[:L], synth.values_f64(tr.Q_pre[l:l + 1], cfg.dtype),
+                             tr.qpos_pre, tr.page_start[:tr.P_pre], tr.page_len[:tr.P_pre])
+        post = oracle.Problem(K, V, tr.pos, synth.values_f64(tr.Q_post[l:l + 1], cfg.dtype), tr.qpos_post,
+                              tr.page_start, tr.page_len)
+        t0 = time.perf_counter()
+        oracle.page_effects(pre, "closed", nthreads=threads)
+        oracle.page_effects(post, "closed", nthreads=threads)
+        elapsed += time.perf_counter() - t0
+        done_layers += 1
+    frac = done_layers / cfg.M
+    tokens = (tr.S_pre + tr.S_post) * frac
+    desc = (f"fp64 closed-form oracle (Eq. 6), pre+post scoring of {done_layers} of {cfg.M} layers "
+            f"(all {cfg.H} KV heads, {cfg.Hq} query heads) of trajectory 0; {elapsed:.1f} s")
+    return tokens / elapsed, threads, desc
+
+
+# ----------------------------------------------------------------------------
+
+
+def algorithmic(cfg):
+    """Scoring roofline terms per token: K and V read once (bytes) and
+    QK^T + PV once (flops), summed over layers and KV heads."""
+    eb = 2 if cfg.dtype == "bf16" else 4
+    bytes_per_tok = cfg.M * cfg.H * 2 * cfg.d * eb
+    flops_per_tok = cfg.M * cfg.H * 4 * cfg.g * cfg.W * cfg.d
+    return bytes_per_tok, flops_per_tok
+
+
+def run_ours(args, rank, world, local):
+    import torch
+
+    from paper_2608_07855_gb300 import commitkv as ck
+    from paper_2608_07855_gb300 import synth
+    from paper_2608_07855_gb300.workload import DeviceTrajectory, StepBuffers
+
+    torch.cuda.set_device(local)
+    cfg = synth.CONFIGS[args.config]
+    n_traj = cfg.n_traj
+    trs = [synth.make_trajectory(cfg, args.seed + 1000 * rank, traj=i) for i in range(n_traj)]
+    devs = [DeviceTrajectory.upload(t) for t in trs]
+    buf = StepBuffers(cfg, devs)
+    stream = torch.cuda.current_stream()
+    tokens_per_step = sum(t.S_pre + t.S_post for t in trs)
+
+    # warm-up
+    for _ in range(args.warmup):
+        buf.step()
+    torch.cuda.synchronize()
+    st = buf.status()
+    if st != ck.COMMITKV_OK:
+        raise RuntimeError(f"device status after warm-up: {ck.status_string(st)}")
+
+    stage_names = ["score_pre", "score_post", "classify", "joint", "compact"]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stage_names) + 1)]
+          for _ in range(args.steps)]
+    clocks = Clocks(local)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        e = ev[k]
+        e[0].record(stream)
+        buf.score_pre()
+        e[1].record(stream)
+        buf.score_post()
+        e[2].record(stream)
+        buf.classify()
+        e[3].record(stream)
+        buf.joint()
+        e[4].record(stream)
+        buf.compact()
+        e[5].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    stage_ms = {n: float(np.mean([ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(args.steps)]))
+                for i, n in enumerate(stage_names)}
+    st = buf.status()
+    if st != ck.COMMITKV_OK:
+        raise RuntimeError(f"device status after timing: {ck.status_string(st)}")
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = tokens_per_step * world / (ms_per_step / 1e3)
+
+    # roofline of the scoring pass (the dominant stage)
+    peaks, peak_kind = load_peaks()
+    bpt, fpt = algorithmic(cfg)
+    score_ms = stage_ms["score_pre"] + stage_ms["score_post"]
+    alg_bytes = bpt * tokens_per_step
+    alg_flops = fpt * tokens_per_step
+    t_mem = alg_bytes / (peaks["hbm_gbs"] * 1e9)
+    t_ten = alg_flops / (peaks["bf16_tflops_sustained"] * 1e12)
+    if t_mem >= t_ten:
+        roof = {"bound": "hbm", "achieved": alg_bytes / (score_ms / 1e3) / 1e9,
+                "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    else:
+        roof = {"bound": "tensor", "achieved": alg_flops / (score_ms / 1e3) / 1e12,
+                "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["kernel"] = "commitkv_page_effects (pre + post scoring passes)"
+    roof["peak_source"] = f"{peak_kind} ({'MEASURED_PEAKS.json' if peak_kind == 'measured' else 'recipe fallback'})"
+    roof["algorithmic_bytes_per_step"] = alg_bytes
+    roof["algorithmic_flops_per_step"] = alg_flops
+    roof["scoring_ms_per_step"] = score_ms
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world)
+
+    result = {
+        "metric": "KV tokens scored/sec (pre+post commit) at Qwen3-8B shape, 32K ctx; % of roofline",
+        "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if cfg.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": cfg.name, "layers": cfg.M, "q_heads": cfg.Hq, "kv_heads": cfg.H,
+                   "head_dim": cfg.d, "L_pre": [t.L_pre for t in trs][:4], "L_obs": [t.L_obs for t in trs][:4],
+                   "window": cfg.W, "page": cfg.G, "budget": cfg.B, "trajectories_per_gpu": n_traj,
+                   "tokens_per_step_per_gpu": tokens_per_step,
+                   "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}"},
+        "stage_ms": stage_ms,
+        "scoring_tokens_per_s": tokens_per_step * world / (score_ms / 1e3),
+        "roofline": roof,
+        "clocks": clk,
+        "gpu_launches": buf_launches(buf) * args.steps,
+    }
+    if e2e:
+        result["e2e"] = e2e
+    return result, cfg, trs
+
+
+def buf_launches(buf):
+    """Kernels of this library launched per step (counted from the launch
+    sequence of each call): scoring = pass A + combine + pass B per cache,
+    classify 1, joint test 1, compaction = select + gather."""
+    return 3 + 3 + 1 + 1 + 2
+
+
+def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):
+    """Same step with inputs copied from pinned host memory each step and the
+    step's decisions (effects, states, accepted pages, retained indices) read
+    back, all inside the timed region."""
+    import torch
+
+    host = []
+    for d in devs:
+        h = {}
+        for name in ("K", "V", "Q_pre", "Q_post", "pos", "page_start", "page_len", "eligible", "pending", "fill"):
+            t = getattr(d, name)
+            h[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True).copy_(t)
+        host.append(h)
+    outs = [[torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in (r_pre, r_post, st, acc, idx)]
+            for r_pre, r_post, st, acc, idx in zip(buf.R_pre, buf.R_post, buf.state, buf.accepted, buf.idx)]
+    n_idx_h = torch.empty(buf.n_idx.shape, dtype=buf.n_idx.dtype, pin_memory=True)
+    h2d = sum(x.numel() * x.element_size() for h in host for x in h.values())
+    d2h = sum(x.numel() * x.element_size() for o in outs for x in o) + n_idx_h.numel() * 4
+    stream = torch.cuda.current_stream()
+    steps = max(2, min(args.steps, 5))
+
+    def one():
+        for d, h in zip(devs, host):
+            for name, x in h.items():
+                getattr(d, name).copy_(x, non_blocking=True)
+        buf.step()
+        for o, srcs in zip(outs, zip(buf.R_pre, buf.R_post, buf.state, buf.accepted, buf.idx)):
+            for dst, src in zip(o, srcs):
+                dst.copy_(src, non_blocking=True)
+        n_idx_h.copy_(buf.n_idx, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        one()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": tokens_per_step * world / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "steps": steps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+def run_reference(args, rank, world):
+    from paper_2608_07855_gb300 import synth
+
+    cfg = synth.CONFIGS[args.config]
+    if rank != 0:
+        return None
+    tr = synth.make_trajectory(cfg, args.seed, traj=0)
+    vals, ts = [], []
+    threads, desc = 1, ""
+    per_step_budget = max(2.0, min(args.cpu_sample_seconds, 120.0 / max(1, args.steps + args.warmup)))
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        v, threads, desc = oracle_sample(cfg, tr, per_step_budget)
+        if k >= args.warmup:
+            vals.append(v)
+            ts.append(time.perf_counter() - t0)
+    value = float(np.median(vals))
+    ms = float(np.mean(ts)) * 1e3
+    return {
+        "impl": "reference", "metric": "KV tokens scored/sec (pre+post commit) at Qwen3-8B shape, 32K ctx; % of roofline",
+        "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "layers": cfg.M, "q_heads": cfg.Hq, "kv_heads": cfg.H,
+                   "head_dim": cfg.d, "L_pre": tr.L_pre, "L_obs": tr.L_obs, "window": cfg.W, "page": cfg.G},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        if args.impl == "ours":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl")
+        else:
+            dist.init_process_group("gloo")
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
+    res, cfg, trs = run_ours(args, rank, world, local)
+    if rank == 0 and not args.no_cpu_baseline:
+        v, threads, desc = oracle_sample(cfg, trs[0], args.cpu_sample_seconds)
+        res["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,423 @@
+// C ABI of the CommitKV hot path: argument checks, workspace layout and
+// launch sequences.  Every entry point is declared in include/commitkv.h.
+#include <math.h>
+#include <string.h>
+
+#include "ckv_internal.cuh"
+
+namespace ckv {
+int simt_rows_per_block();
+int simt_pages_per_block();
+int joint_rows_per_group();
+int compact_max_pending();
+}  // namespace ckv
+
+using namespace ckv;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+int layers_selected(const commitkv_shape *s, const uint8_t *mask, uint8_t *ids) {
+  int n = 0;
+  for (int l = 0; l < s->layers; ++l)
+    if (!mask || mask[l]) ids[n++] = (uint8_t)l;
+  return n;
+}
+
+commitkv_status check_shape(const commitkv_shape *s) {
+  if (!s) return COMMITKV_ERR_INVALID_ARG;
+  if (s->layers < 1 || s->layers > kMaxLayers || s->kv_heads < 1 || s->q_heads < s->kv_heads ||
+      s->q_heads % s->kv_heads != 0 || s->head_dim < 1)
+    return COMMITKV_ERR_INVALID_ARG;
+  if (s->dtype != COMMITKV_F32 && s->dtype != COMMITKV_BF16) return COMMITKV_ERR_INVALID_ARG;
+  if (!(s->softmax_scale >= 0.0f) || isinf(s->softmax_scale)) return COMMITKV_ERR_INVALID_ARG;
+  if (s->head_dim != 64 && s->head_dim != 128) return COMMITKV_ERR_UNSUPPORTED;
+  if ((int64_t)s->layers * s->q_heads > (1 << 20)) return COMMITKV_ERR_INVALID_ARG;
+  return COMMITKV_OK;
+}
+
+commitkv_status check_trajs(const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
+                            bool need_q) {
+  if (n_traj < 1 || n_traj > kMaxTraj || !tr) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t) {
+    const commitkv_traj &x = tr[t];
+    if (x.S < 0 || x.W < 0 || x.P < 0) return COMMITKV_ERR_INVALID_ARG;
+    if (x.S > 0 && (!x.k || !x.v || !x.pos)) return COMMITKV_ERR_INVALID_ARG;
+    if (x.P > 0 && (!x.page_start || !x.page_len)) return COMMITKV_ERR_INVALID_ARG;
+    if (need_q && x.W > 0 && (!x.q || !x.q_pos)) return COMMITKV_ERR_INVALID_ARG;
+    if (x.stride_tok < s->head_dim || x.stride_head < 0 || x.stride_layer < 0)
+      return COMMITKV_ERR_INVALID_ARG;
+    if ((int64_t)(s->q_heads / s->kv_heads) * x.W > (1 << 24)) return COMMITKV_ERR_INVALID_ARG;
+  }
+  return COMMITKV_OK;
+}
+
+TrajDev to_dev(const commitkv_traj &x) {
+  TrajDev d;
+  d.k = x.k;
+  d.v = x.v;
+  d.sl = x.stride_layer;
+  d.sh = x.stride_head;
+  d.st = x.stride_tok;
+  d.pos = x.pos;
+  d.q = x.q;
+  d.qpos = x.q_pos;
+  d.ps = x.page_start;
+  d.pl = x.page_len;
+  d.S = x.S;
+  d.W = x.W;
+  d.P = x.P;
+  d.pad = 0;
+  return d;
+}
+
+void fill_batch(Batch &b, const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
+                const uint8_t *mask) {
+  memset(&b, 0, sizeof b);
+  b.n_traj = n_traj;
+  b.M = s->layers;
+  b.H = s->kv_heads;
+  b.Hq = s->q_heads;
+  b.g = s->q_heads / s->kv_heads;
+  b.d = s->head_dim;
+  b.dtype = s->dtype;
+  b.scale = s->softmax_scale > 0.0f ? s->softmax_scale : 1.0f / sqrtf((float)s->head_dim);
+  b.scale_log2 = b.scale * 1.4426950408889634f;
+  b.n_layers = layers_selected(s, mask, b.layer_ids);
+  for (int t = 0; t < n_traj; ++t) b.t[t] = to_dev(tr[t]);
+}
+
+int chunk_len_for(int n_traj, const commitkv_traj *tr) {
+  int smax = 0;
+  for (int t = 0; t < n_traj; ++t) smax = tr[t].S > smax ? tr[t].S : smax;
+  int c = (smax + 15) / 16;
+  if (c < 512) c = 512;
+  return (c + 63) / 64 * 64;
+}
+
+int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// Region sizes of each call (bytes after the 256-byte header).
+size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, int n_layers) {
+  int CL = chunk_len_for(n_traj, tr), RB = simt_rows_per_block(), d = s->head_dim;
+  int g = s->q_heads / s->kv_heads;
+  size_t units = 0, stats = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    int rows = g * tr[t].W;
+    units += (size_t)n_layers * s->kv_heads * cdiv(tr[t].S, CL) * cdiv(rows, RB);
+    stats += align_up((size_t)s->layers * s->q_heads * tr[t].W * (d + 4) * 4);
+  }
+  return align_up(units * RB * (d + 4) * 4) + stats;
+}
+
+size_t joint_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, int n_layers) {
+  int g = s->q_heads / s->kv_heads, d = s->head_dim;
+  size_t rows = 0, steps = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    rows += (size_t)n_layers * s->kv_heads * g * tr[t].W;
+    steps += align_up((size_t)tr[t].P * 4);
+  }
+  return 2 * align_up(rows * d * 4) + align_up(rows * 16) + steps;
+}
+
+size_t classify_bytes(int n_traj, const int32_t *P) {
+  size_t b = 0;
+  for (int t = 0; t < n_traj; ++t) b += align_up((size_t)P[t] * 4);
+  return b;
+}
+
+size_t compact_bytes(int n_traj, const commitkv_traj *tr) {
+  size_t b = 0;
+  for (int t = 0; t < n_traj; ++t) b += align_up((size_t)tr[t].S);
+  return b;
+}
+
+commitkv_status check_ws(void *ws, size_t bytes, size_t need) {
+  if (!ws || ((uintptr_t)ws % kAlign) != 0) return COMMITKV_ERR_WORKSPACE;
+  if (bytes < need) return COMMITKV_ERR_WORKSPACE;
+  return COMMITKV_OK;
+}
+
+commitkv_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return COMMITKV_OK;
+  cudaGetLastError();  // clear the sticky-free error state of this thread
+  return COMMITKV_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t commitkv_workspace_size(const commitkv_shape *shape, int32_t n_traj,
+                               const commitkv_traj *trajs) {
+  if (check_shape(shape) != COMMITKV_OK) return 0;
+  if (check_trajs(shape, n_traj, trajs, false) != COMMITKV_OK) return 0;
+  int32_t P[kMaxTraj];
+  for (int t = 0; t < n_traj; ++t) P[t] = trajs[t].P;
+  size_t need = score_bytes(shape, n_traj, trajs, shape->layers);
+  size_t j = joint_bytes(shape, n_traj, trajs, shape->layers);
+  size_t c = classify_bytes(n_traj, P);
+  size_t k = compact_bytes(n_traj, trajs);
+  if (j > need) need = j;
+  if (c > need) need = c;
+  if (k > need) need = k;
+  return kAlign + need;
+}
+
+commitkv_status commitkv_workspace_init(void *workspace, size_t workspace_bytes,
+                                        cudaStream_t stream) {
+  if (!workspace || workspace_bytes < kAlign || ((uintptr_t)workspace % kAlign)) return COMMITKV_ERR_WORKSPACE;
+  return cuda_status(cudaMemsetAsync(workspace, 0, sizeof(WsHeader), stream));
+}
+
+commitkv_status commitkv_workspace_status(const void *workspace, size_t workspace_bytes,
+                                          cudaStream_t stream, int32_t clear) {
+  if (!workspace || workspace_bytes < kAlign || ((uintptr_t)workspace % kAlign)) return COMMITKV_ERR_WORKSPACE;
+  WsHeader h;
+  cudaError_t e = cudaMemcpyAsync(&h, workspace, sizeof h, cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (clear) {
+    e = cudaMemsetAsync(const_cast<void *>(workspace), 0, sizeof(WsHeader), stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return (commitkv_status)h.status;
+}
+
+const char *commitkv_status_string(commitkv_status s) {
+  switch (s) {
+    case COMMITKV_OK: return "ok";
+    case COMMITKV_ERR_INVALID_ARG: return "invalid argument";
+    case COMMITKV_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case COMMITKV_ERR_CUDA: return "CUDA runtime error";
+    case COMMITKV_ERR_TIMEOUT: return "bounded device wait timed out";
+    case COMMITKV_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+    case COMMITKV_ERR_DEVICE_INPUT: return "device-resident input failed a device-side check";
+  }
+  return "unknown status";
+}
+
+commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_traj,
+                                      const commitkv_traj *trajs, const uint8_t *layer_mask,
+                                      float *const *R_out, float *const *head_R_out,
+                                      float *const *stats_out, void *workspace,
+                                      size_t workspace_bytes, cudaStream_t stream) {
+  commitkv_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_trajs(shape, n_traj, trajs, true))) return st;
+  if (!R_out) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t)
+    if (trajs[t].P > 0 && !R_out[t]) return COMMITKV_ERR_INVALID_ARG;
+
+  static thread_local ScoreLaunch L;  // large: keep off the stack
+  memset(&L, 0, sizeof L);
+  fill_batch(L.batch, shape, n_traj, trajs, layer_mask);
+  int nl = L.batch.n_layers;
+  size_t need = kAlign + score_bytes(shape, n_traj, trajs, shape->layers);
+  if ((st = check_ws(workspace, workspace_bytes, need))) return st;
+
+  int CL = chunk_len_for(n_traj, trajs), RB = simt_rows_per_block(), PG = simt_pages_per_block();
+  int g = L.batch.g, d = shape->head_dim;
+  L.chunk_len = CL;
+  char *base = static_cast<char *>(workspace) + kAlign;
+  size_t units = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    int rows = g * trajs[t].W;
+    L.nrb[t] = cdiv(rows, RB);
+    L.nchunk[t] = cdiv(trajs[t].S, CL);
+    L.npg[t] = cdiv(trajs[t].P, PG);
+    L.unit_off_a[t + 1] = L.unit_off_a[t] + nl * shape->kv_heads * L.nchunk[t] * L.nrb[t];
+    L.unit_off_b[t + 1] = L.unit_off_b[t] + nl * shape->kv_heads * L.npg[t] * L.nrb[t];
+    L.row_off[t + 1] = L.row_off[t] + nl * shape->kv_heads * rows;
+    units += (size_t)nl * shape->kv_heads * L.nchunk[t] * L.nrb[t];
+  }
+  float *partials = reinterpret_cast<float *>(base);
+  char *sbase = base + align_up(units * RB * (d + 4) * 4);
+  // (the layout is computed for every layer; a mask only uses a prefix)
+  size_t full_units = 0;
+  for (int t = 0; t < n_traj; ++t)
+    full_units += (size_t)shape->layers * shape->kv_heads * L.nchunk[t] * L.nrb[t];
+  sbase = base + align_up(full_units * RB * (d + 4) * 4);
+  for (int t = 0; t < n_traj; ++t) {
+    size_t sb = align_up((size_t)shape->layers * shape->q_heads * trajs[t].W * (d + 4) * 4);
+    L.stats[t] = (stats_out && stats_out[t]) ? stats_out[t] : reinterpret_cast<float *>(sbase);
+    sbase += sb;
+    L.R[t] = R_out[t];
+    L.headR[t] = head_R_out ? head_R_out[t] : nullptr;
+  }
+  for (int t = 0; t < n_traj; ++t) {
+    if (trajs[t].P == 0) continue;
+    cudaError_t e = cudaMemsetAsync(R_out[t], 0, (size_t)trajs[t].P * 4, stream);
+    if (e == cudaSuccess && L.headR[t])
+      e = cudaMemsetAsync(L.headR[t], 0, (size_t)shape->layers * shape->q_heads * trajs[t].P * 4, stream);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  WsHeader *hdr = static_cast<WsHeader *>(workspace);
+  return cuda_status(launch_score_simt(L, partials, hdr, stream));
+}
+
+commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float *const *R_pre,
+                                  const float *const *R_post, const uint8_t *const *eligible,
+                                  const commitkv_thresholds *thresholds, uint8_t *const *state_out,
+                                  int32_t *const *cand_out, int32_t *n_cand_out, void *workspace,
+                                  size_t workspace_bytes, cudaStream_t stream) {
+  if (n_traj < 1 || n_traj > kMaxTraj || !P || !R_pre || !R_post || !eligible || !state_out ||
+      !cand_out || !n_cand_out)
+    return COMMITKV_ERR_INVALID_ARG;
+  commitkv_thresholds th = thresholds ? *thresholds : commitkv_thresholds{0.05f, 0.01f, 0.75f, 0.25f};
+  if (!(th.tau_dead < th.tau_use) || !(th.rho_dead < th.rho_use)) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t) {
+    if (P[t] < 0) return COMMITKV_ERR_INVALID_ARG;
+    if (P[t] > 0 && (!R_pre[t] || !R_post[t] || !eligible[t] || !state_out[t] || !cand_out[t]))
+      return COMMITKV_ERR_INVALID_ARG;
+  }
+  commitkv_status st = check_ws(workspace, workspace_bytes, kAlign + classify_bytes(n_traj, P));
+  if (st) return st;
+  ClassifyLaunch L;
+  memset(&L, 0, sizeof L);
+  L.n_traj = n_traj;
+  char *base = static_cast<char *>(workspace) + kAlign;
+  for (int t = 0; t < n_traj; ++t) {
+    L.P[t] = P[t];
+    L.Rm[t] = R_pre[t];
+    L.Rp[t] = R_post[t];
+    L.el[t] = eligible[t];
+    L.state[t] = state_out[t];
+    L.cand[t] = cand_out[t];
+    L.scratch[t] = reinterpret_cast<int32_t *>(base);
+    base += align_up((size_t)P[t] * 4);
+  }
+  L.n_cand = n_cand_out;
+  L.tau_use = th.tau_use;
+  L.tau_dead = th.tau_dead;
+  L.rho_use = (double)th.rho_use;
+  L.rho_dead = (double)th.rho_dead;
+  return cuda_status(launch_classify(L, static_cast<WsHeader *>(workspace), stream));
+}
+
+commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
+                                    const commitkv_traj *post, const uint8_t *layer_mask,
+                                    const float *const *stats, const int32_t *const *cand,
+                                    const int32_t *n_cand, float tau_joint,
+                                    uint8_t *const *accepted_out, float *const *step_R_out,
+                                    void *workspace, size_t workspace_bytes,
+                                    cudaStream_t stream) {
+  commitkv_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_trajs(shape, n_traj, post, true))) return st;
+  if (!stats || !cand || !n_cand || !accepted_out || isnan(tau_joint)) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t)
+    if (post[t].P > 0 && (!stats[t] || !cand[t] || !accepted_out[t])) return COMMITKV_ERR_INVALID_ARG;
+  size_t need = kAlign + joint_bytes(shape, n_traj, post, shape->layers);
+  if ((st = check_ws(workspace, workspace_bytes, need))) return st;
+
+  static thread_local JointLaunch L;
+  memset(&L, 0, sizeof L);
+  fill_batch(L.batch, shape, n_traj, post, layer_mask);
+  int nl = L.batch.n_layers, g = L.batch.g, d = shape->head_dim, RB = joint_rows_per_group();
+  size_t rows_total = 0;
+  int maxP = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    int rows = g * post[t].W;
+    L.nrb[t] = cdiv(rows, RB);
+    L.group_off[t + 1] = L.group_off[t] + nl * shape->kv_heads * L.nrb[t];
+    L.row_off[t + 1] = L.row_off[t] + nl * shape->kv_heads * rows;
+    rows_total += (size_t)nl * shape->kv_heads * rows;
+    maxP = post[t].P > maxP ? post[t].P : maxP;
+  }
+  size_t rows_full = 0;
+  for (int t = 0; t < n_traj; ++t) rows_full += (size_t)shape->layers * shape->kv_heads * g * post[t].W;
+  char *base = static_cast<char *>(workspace) + kAlign;
+  L.DA = reinterpret_cast<float *>(base);
+  base += align_up(rows_full * d * 4);
+  L.DE = reinterpret_cast<float *>(base);
+  base += align_up(rows_full * d * 4);
+  L.SA = reinterpret_cast<float *>(base);
+  base += align_up(rows_full * 16);
+  char *step_base = base;
+  for (int t = 0; t < n_traj; ++t) {
+    L.stats[t] = stats[t];
+    L.cand[t] = cand[t];
+    L.accepted[t] = accepted_out[t];
+    L.stepR_out[t] = step_R_out ? step_R_out[t] : nullptr;
+    L.stepR[t] = reinterpret_cast<float *>(base);
+    base += align_up((size_t)post[t].P * 4);
+  }
+  L.n_cand = n_cand;
+  L.tau = tau_joint;
+  L.max_steps = maxP;
+  cudaError_t e = cudaMemsetAsync(L.DA, 0, rows_total * d * 4, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L.SA, 0, rows_full * 16, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(step_base, 0, (size_t)(base - step_base), stream);
+  for (int t = 0; t < n_traj && e == cudaSuccess; ++t)
+    if (post[t].P > 0) e = cudaMemsetAsync(accepted_out[t], 0, post[t].P, stream);
+  // the barrier counters start from a known state
+  WsHeader *hdr = static_cast<WsHeader *>(workspace);
+  if (e == cudaSuccess) e = cudaMemsetAsync(&hdr->abort, 0, 3 * sizeof(int32_t), stream);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (rows_total == 0 || maxP == 0) return COMMITKV_OK;
+  int dev = 0, sms = 0;
+  e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_status(e);
+  return cuda_status(launch_joint(L, hdr, stream, sms));
+}
+
+commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
+                                 const commitkv_traj *cache, const uint8_t *const *retired,
+                                 const int32_t *const *pending, const int32_t *n_pending,
+                                 const float *const *pending_priority,
+                                 const float *const *fill_score, int32_t budget_B,
+                                 int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                 int32_t *const *idx_out, int32_t *n_idx_out,
+                                 void *const *k_out, void *const *v_out, int32_t *const *pos_out,
+                                 void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+  commitkv_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_trajs(shape, n_traj, cache, false))) return st;
+  if (budget_B < 0 || pending_tokens_BN < 0 || pending_tokens_BN > budget_B || pending_cap_pages < 0)
+    return COMMITKV_ERR_INVALID_ARG;
+  if (!retired || !n_pending || !fill_score || !idx_out || !n_idx_out) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t) {
+    if (n_pending[t] < 0 || n_pending[t] > compact_max_pending()) return COMMITKV_ERR_INVALID_ARG;
+    if (n_pending[t] > 0 && (!pending || !pending[t] || !pending_priority || !pending_priority[t]))
+      return COMMITKV_ERR_INVALID_ARG;
+    if (cache[t].P > 0 && !retired[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (cache[t].S > 0 && !fill_score[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (budget_B > 0 && !idx_out[t]) return COMMITKV_ERR_INVALID_ARG;
+  }
+  if ((st = check_ws(workspace, workspace_bytes, kAlign + compact_bytes(n_traj, cache)))) return st;
+  static thread_local CompactLaunch L;
+  memset(&L, 0, sizeof L);
+  L.n_traj = n_traj;
+  L.M = shape->layers;
+  L.H = shape->kv_heads;
+  L.d = shape->head_dim;
+  L.elem_bytes = shape->dtype == COMMITKV_BF16 ? 2 : 4;
+  char *base = static_cast<char *>(workspace) + kAlign;
+  for (int t = 0; t < n_traj; ++t) {
+    L.t[t] = to_dev(cache[t]);
+    L.retired[t] = retired[t];
+    L.pending[t] = n_pending[t] ? pending[t] : nullptr;
+    L.n_pending[t] = n_pending[t];
+    L.prio[t] = n_pending[t] ? pending_priority[t] : nullptr;
+    L.fill[t] = fill_score[t];
+    L.cls[t] = reinterpret_cast<uint8_t *>(base);
+    base += align_up((size_t)cache[t].S);
+    L.idx[t] = idx_out[t];
+    L.k_out[t] = k_out ? k_out[t] : nullptr;
+    L.v_out[t] = v_out ? v_out[t] : nullptr;
+    L.pos_out[t] = pos_out ? pos_out[t] : nullptr;
+  }
+  L.n_idx = n_idx_out;
+  L.B = budget_B;
+  L.B_N = pending_tokens_BN;
+  L.cap = pending_cap_pages;
+  return cuda_status(launch_compact(L, static_cast<WsHeader *>(workspace), stream));
+}
+
+}  // extern "C"

@@ -266,11 +266,14 @@ class Trajectory:
 
     @property
     def qpos_pre(self):
-        return np.arange(self.L_pre - self.cfg.W, self.L_pre, dtype=np.int32)
+        """Q-c: the positions of the last W tokens of y_t (Eq. 5)."""
+        return np.ascontiguousarray(self.pos[self.L_pre - self.cfg.W: self.L_pre], np.int32)
 
     @property
     def qpos_post(self):
-        return np.arange(self.L_pre + self.L_obs, self.L_pre + self.L_obs + self.cfg.W, dtype=np.int32)
+        """Q+c: the positions of the first W decoded tokens after o_t (Eq. 5)."""
+        b = self.L_pre + self.L_obs
+        return np.ascontiguousarray(self.pos[b: b + self.cfg.W], np.int32)
 
     @property
     def P_post(self):
@@ -355,6 +358,7 @@ def make_trajectory(cfg: Config, seed: int = 0, traj: int = 0, values: bool = Tr
     planted = np.asarray([pool[i] for i in planted], np.int32)
     tr = Trajectory(cfg, seed, traj, L_pre, L_obs, ev, ps, pl, pe, P_pre, eligible, planted)
     tr.pending = np.asarray([E for E in range(len(ps)) if pe[E] == len(ev) - 2], np.int32)
+    tr.pos = np.arange(tr.S_post, dtype=np.int32)
     if values:
         _fill_values(tr)
     return tr
@@ -370,7 +374,6 @@ def _fill_values(tr: Trajectory):
     tr.V = np.empty((M, H, S, d), dt)
     Qpre = np.empty((M, Hq, W, d), np.float32)
     Qpost = np.empty((M, Hq, W, d), np.float32)
-    tr.pos = np.arange(S, dtype=np.int32)
     tr.fill_score = uniform_array(seed, _stream(t, _T_FILL), S)
     plant_tok = np.concatenate([np.arange(tr.page_start[E], tr.page_start[E] + tr.page_len[E])
                                 for E in tr.planted]) if len(tr.planted) else np.zeros(0, np.int64)

@@ -1,0 +1,96 @@
+"""The C-ABI library builds for sm_103a, loads, exports every entry point the
+header declares, and rejects bad arguments on the host (no GPU needed: none
+of these calls reaches the device)."""
+import ctypes
+
+import pytest
+
+from paper_2608_07855_gb300 import build, commitkv as ck
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return ck.load_library()
+
+
+def test_header_declares_the_entry_points():
+    names = ck.declared_functions()
+    for n in ("commitkv_page_effects", "commitkv_classify", "commitkv_joint_test", "commitkv_compact",
+              "commitkv_workspace_size", "commitkv_workspace_init", "commitkv_workspace_status",
+              "commitkv_status_string"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in ck.declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    for s in range(7):
+        assert ck.status_string(s) and ck.status_string(s) != "unknown status"
+    assert ck.status_string(99) == "unknown status"
+
+
+def _good_traj(S=100, W=8, P=4, d=128, H=2):
+    return ck.Traj(0x10000, 0x20000, H * S * d, S * d, d, 0x30000, S, 0x40000, 0x50000, W, 0x60000,
+                   0x70000, P)
+
+
+def test_workspace_size_host_only(lib):
+    shape = ck.Shape(2, 2, 8, 128, ck.COMMITKV_BF16, 0.0)
+    trajs = (ck.Traj * 1)(_good_traj())
+    n = lib.commitkv_workspace_size(ctypes.byref(shape), 1, trajs)
+    assert n > 256 and n % 256 == 0
+    bad = ck.Shape(2, 3, 8, 128, ck.COMMITKV_BF16, 0.0)  # Hq not a multiple of H
+    assert lib.commitkv_workspace_size(ctypes.byref(bad), 1, trajs) == 0
+    assert lib.commitkv_workspace_size(ctypes.byref(shape), 0, trajs) == 0
+    assert lib.commitkv_workspace_size(ctypes.byref(shape), 65, trajs) == 0
+
+
+def test_host_validation(lib):
+    shape = ck.Shape(2, 2, 8, 128, ck.COMMITKV_BF16, 0.0)
+    trajs = (ck.Traj * 1)(_good_traj())
+    R = (ctypes.c_void_p * 1)(0x80000)
+    f = lib.commitkv_page_effects
+    # unsupported head width
+    s96 = ck.Shape(2, 2, 8, 96, ck.COMMITKV_BF16, 0.0)
+    assert f(ctypes.byref(s96), 1, trajs, None, R, None, None, 0x90000, 1 << 30, None) == ck.COMMITKV_ERR_UNSUPPORTED
+    # bad dtype, bad scale
+    for bad in (ck.Shape(2, 2, 8, 128, 7, 0.0), ck.Shape(2, 2, 8, 128, 1, -1.0), ck.Shape(0, 2, 8, 128, 1, 0.0)):
+        assert f(ctypes.byref(bad), 1, trajs, None, R, None, None, 0x90000, 1 << 30, None) == ck.COMMITKV_ERR_INVALID_ARG
+    # missing outputs
+    assert f(ctypes.byref(shape), 1, trajs, None, None, None, None, 0x90000, 1 << 30, None) == ck.COMMITKV_ERR_INVALID_ARG
+    # missing / small / misaligned workspace
+    assert f(ctypes.byref(shape), 1, trajs, None, R, None, None, None, 1 << 30, None) == ck.COMMITKV_ERR_WORKSPACE
+    assert f(ctypes.byref(shape), 1, trajs, None, R, None, None, 0x90000, 1024, None) == ck.COMMITKV_ERR_WORKSPACE
+    assert f(ctypes.byref(shape), 1, trajs, None, R, None, None, 0x90001, 1 << 30, None) == ck.COMMITKV_ERR_WORKSPACE
+    # negative sizes, null pointers with work to do
+    for kw in (dict(S=-1), dict(W=-1), dict(P=-1)):
+        t = (ck.Traj * 1)(_good_traj(**{**dict(S=100, W=8, P=4), **kw}))
+        assert f(ctypes.byref(shape), 1, t, None, R, None, None, 0x90000, 1 << 30, None) == ck.COMMITKV_ERR_INVALID_ARG
+    t = _good_traj()
+    t.k = None
+    assert f(ctypes.byref(shape), 1, (ck.Traj * 1)(t), None, R, None, None, 0x90000, 1 << 30, None) == ck.COMMITKV_ERR_INVALID_ARG
+
+
+def test_classify_and_compact_validation(lib):
+    P = (ctypes.c_int32 * 1)(10)
+    ptrs = (ctypes.c_void_p * 1)(0x1000)
+    th = ck.Thresholds(0.01, 0.05, 0.75, 0.25)  # tau_dead > tau_use
+    assert lib.commitkv_classify(1, P, ptrs, ptrs, ptrs, ctypes.byref(th), ptrs, ptrs, 0x2000, 0x90000, 1 << 20, None) \
+        == ck.COMMITKV_ERR_INVALID_ARG
+    th = ck.Thresholds(0.05, 0.01, 0.25, 0.75)  # rho_dead > rho_use
+    assert lib.commitkv_classify(1, P, ptrs, ptrs, ptrs, ctypes.byref(th), ptrs, ptrs, 0x2000, 0x90000, 1 << 20, None) \
+        == ck.COMMITKV_ERR_INVALID_ARG
+    shape = ck.Shape(2, 2, 8, 128, ck.COMMITKV_BF16, 0.0)
+    trajs = (ck.Traj * 1)(_good_traj())
+    npend = (ctypes.c_int32 * 1)(0)
+    # B_N > B
+    assert lib.commitkv_compact(ctypes.byref(shape), 1, trajs, ptrs, None, npend, None, ptrs, 10, 11, 4,
+                                ptrs, 0x3000, None, None, None, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
+    # too many pending pages
+    npend = (ctypes.c_int32 * 1)(100000)
+    assert lib.commitkv_compact(ctypes.byref(shape), 1, trajs, ptrs, ptrs, npend, ptrs, ptrs, 10, 5, 4,
+                                ptrs, 0x3000, None, None, None, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG

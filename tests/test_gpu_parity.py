@@ -1,0 +1,350 @@
+"""GPU parity of the CommitKV library against the CPU oracle.
+
+Every test calls the CUDA path through the C ABI (the Python binding only
+marshals pointers) on seeded synthetic inputs and compares element by
+element with the oracle on the same inputs:
+  effects R-, R+ and per-(layer, head) maxima: 1e-4 relative for fp32 inputs,
+  2e-2 relative for bf16 inputs (fp32 accumulation), infinities and zeros
+  exact;
+  classification and ordering: bit-exact on the same fp32 effects;
+  joint test: step effects within the effect tolerance, and the accepted
+  set identical up to the first step whose decision margin |R - tau| / tau
+  is within that tolerance;
+  selection, gather and positions: bit-exact.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import core  # noqa: E402
+from paper_2608_07855_gb300 import commitkv as ck  # noqa: E402
+from paper_2608_07855_gb300 import synth  # noqa: E402
+from paper_2608_07855_gb300.workload import DeviceTrajectory, StepBuffers  # noqa: E402
+
+from oracle_bridge import (OracleStep, gapped_positions, isclose_tol, rel_close,  # noqa: E402
+                           safe_threshold_mask)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    ck.load_library()
+
+
+def _cfg(name):
+    if name == "tiny":
+        return synth.CONFIGS["tiny"]
+    if name == "small":
+        return synth.small_config()
+    if name == "small_w40_g16":  # 160 rows per (layer, KV head): ragged row blocks; G = 16
+        return synth.small_config("small_w40_g16", W=40, G=16, L_pre=600, L_obs=70, B=256)
+    if name == "small_f32":
+        return synth.small_config("small_f32", dtype="f32", d=64, H=2, Hq=4, M=1, W=16, G=16,
+                                  L_pre=500, L_obs=60, B=200, outlier_channels=0)
+    if name == "small_long_pages":  # pages longer than one 64-token tile
+        return synth.small_config("small_long_pages", G=100, L_pre=900, L_obs=80, B=400)
+    raise KeyError(name)
+
+
+CASES = [("tiny", 0), ("tiny", 1), ("small", 0), ("small", 1), ("small_w40_g16", 2),
+         ("small_f32", 3), ("small_long_pages", 4)]
+
+
+class Run:
+    """GPU step and oracle step on the same trajectory."""
+
+    def __init__(self, name, seed, gapped=False):
+        cfg = _cfg(name)
+        tr = synth.make_trajectory(cfg, seed)
+        if gapped:
+            gapped_positions(tr, seed)
+        self.cfg, self.tr = cfg, tr
+        self.dev = DeviceTrajectory.upload(tr)
+        self.buf = StepBuffers(cfg, [self.dev])
+        self.orc = OracleStep(tr, "explicit")
+        self.tol = isclose_tol(cfg.dtype)
+
+
+_runs = {}
+
+
+def get_run(name, seed, gapped=False):
+    key = (name, seed, gapped)
+    if key not in _runs:
+        _runs[key] = Run(name, seed, gapped)
+    return _runs[key]
+
+
+def _np(t):
+    return t.detach().cpu().numpy()
+
+
+def _assert_close(got, want, tol, what):
+    ok = rel_close(got, want, tol)
+    if not ok.all():
+        bad = np.flatnonzero(~ok.ravel())[:8]
+        g, w = np.ravel(got), np.ravel(want)
+        raise AssertionError(f"{what}: {int((~ok).sum())} of {ok.size} outside {tol}: "
+                             + ", ".join(f"[{i}] gpu {g[i]:.6g} oracle {w[i]:.6g}" for i in bad))
+
+
+@pytest.mark.parametrize("name,seed", CASES)
+def test_page_effects(name, seed):
+    r = get_run(name, seed)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    headR_pre = torch.zeros(cfg.M, cfg.Hq, dev.P_pre, device="cuda")
+    headR_post = torch.zeros(cfg.M, cfg.Hq, dev.P_post, device="cuda")
+    R_pre = torch.zeros(dev.P_pre, device="cuda")
+    ck.commitkv_page_effects(b.shape, [dev.pre()], [R_pre], head_R_out=[headR_pre], workspace=b.ws)
+    ck.commitkv_page_effects(b.shape, [dev.post()], b.R_post, head_R_out=[headR_post],
+                             stats_out=b.stats, workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    o = r.orc
+    _assert_close(_np(R_pre), o.R_pre[:dev.P_pre], r.tol, "R-")
+    _assert_close(_np(b.R_post[0]), o.R_post, r.tol, "R+")
+    _assert_close(_np(headR_pre), o.H_pre, r.tol, "R- per head")
+    _assert_close(_np(headR_post), o.H_post, r.tol, "R+ per head")
+    # stats: m, l, n, o of every post-commit probe row
+    m, l, o_vec, n = o.stats
+    st = _np(b.stats[0]).reshape(-1, cfg.d + 4)
+    assert np.array_equal(st[:, 2].astype(np.int64), n)
+    _assert_close(st[:, 0], m, 1e-5, "row max")
+    _assert_close(st[:, 1], l, 1e-4, "row sum")
+    err = np.linalg.norm(st[:, 4:] - o_vec, axis=1) / np.maximum(np.linalg.norm(o_vec, axis=1), 1e-30)
+    assert err.max() <= 1e-4, err.max()
+
+
+@pytest.mark.parametrize("name,seed", CASES)
+def test_classify_isolated(name, seed):
+    """Oracle effects (rounded to fp32) into the GPU classifier: states and
+    candidate order must equal the oracle's classification of the same fp32
+    values, bit for bit."""
+    r = get_run(name, seed)
+    b, dev, o = r.buf, r.dev, r.orc
+    Rm = torch.from_numpy(o.R_pre32).cuda()
+    Rp = torch.from_numpy(o.R_post32).cuda()
+    ck.commitkv_classify([dev.P_post], [Rm], [Rp], [dev.eligible], b.state, b.cand, b.n_cand, b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    assert np.array_equal(_np(b.state[0]), o.state)
+    nc = int(b.n_cand[0])
+    assert nc == len(o.cand)
+    assert np.array_equal(_np(b.cand[0])[:nc], o.cand)
+
+
+@pytest.mark.parametrize("name,seed", CASES)
+def test_joint_isolated(name, seed):
+    """The oracle's candidate list into the GPU joint test (with the GPU's
+    own post-commit stats); compare each step's joint effect and the
+    accepted set up to the first decision inside the tolerance."""
+    r = get_run(name, seed)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    b.score_post()
+    cand = torch.zeros(max(dev.P_post, 1), dtype=torch.int32, device="cuda")
+    cand[:len(o.cand)] = torch.from_numpy(o.cand.astype(np.int32)).cuda()
+    n_cand = torch.tensor([len(o.cand)], dtype=torch.int32, device="cuda")
+    ck.commitkv_joint_test(b.shape, [dev.post()], b.stats, [cand], n_cand, cfg.tau_joint, b.accepted,
+                           b.step_R, workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    nc = len(o.cand)
+    step = _np(b.step_R[0])[:nc]
+    acc = _np(b.accepted[0])[:dev.P_post]
+    # compare up to (and including) the first unsafe decision
+    safe = safe_threshold_mask(o.step_R, cfg.tau_joint, r.tol)
+    upto = nc if safe.all() else int(np.argmin(safe))
+    _assert_close(step[:upto], o.step_R[:upto], r.tol, "joint step R")
+    for j in range(upto):
+        E = o.cand[j]
+        assert acc[E] == o.accepted[E], (j, E, step[j], o.step_R[j])
+    # decisions agree with the reported effects everywhere
+    for j in range(nc):
+        assert acc[o.cand[j]] == (step[j] <= cfg.tau_joint)
+    # only candidates can be accepted
+    others = np.setdiff1d(np.arange(dev.P_post), o.cand)
+    assert not acc[others].any()
+
+
+@pytest.mark.parametrize("name,seed", CASES)
+def test_compact_isolated(name, seed):
+    """Same retired set, pending pages, priorities and fill scores into the
+    GPU checkpoint: I_j, K~, V~, p~ bit-exact."""
+    r = get_run(name, seed)
+    cfg, b, dev, o, tr = r.cfg, r.buf, r.dev, r.orc, r.tr
+    retired = torch.from_numpy(o.accepted.astype(np.uint8)).cuda()
+    prio = torch.from_numpy(o.R_post32).cuda()
+    ck.commitkv_compact(b.shape, [dev.post()], [retired], [dev.pending], [prio], [dev.fill], cfg.B,
+                        cfg.B_N, cfg.pending_cap, b.idx, b.n_idx, b.k_out, b.v_out, b.pos_out,
+                        workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    n = int(b.n_idx[0])
+    assert n == len(o.I)
+    I = _np(b.idx[0])[:n]
+    assert np.array_equal(I, o.I)
+    Kw, Vw, pw = core.gather(tr.K, tr.V, tr.pos, o.I)
+    kg = b.k_out[0][:, :, :n]
+    vg = b.v_out[0][:, :, :n]
+    if cfg.dtype == "bf16":
+        kg, vg = kg.view(torch.uint16), vg.view(torch.uint16)
+    assert np.array_equal(_np(kg), Kw) and np.array_equal(_np(vg), Vw)
+    assert np.array_equal(_np(b.pos_out[0])[:n], pw)
+
+
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("small", 1), ("small_f32", 3)])
+def test_full_step(name, seed):
+    """The whole launch sequence of one step: every decision of the GPU
+    pipeline whose margin is safe matches the oracle pipeline."""
+    r = get_run(name, seed)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    b.step()
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    _assert_close(_np(b.R_pre[0]), o.R_pre, r.tol, "R-")
+    _assert_close(_np(b.R_post[0]), o.R_post, r.tol, "R+")
+    st = _np(b.state[0])
+    # classification agrees on pages whose thresholds are not within tolerance
+    from oracle_bridge import percentile_safe
+    idx = np.flatnonzero(dev.tr.eligible)
+    safe = percentile_safe(o.R_pre, idx, r.tol) & percentile_safe(o.R_post, idx, r.tol)
+    for th in (0.05, 0.01):
+        safe &= safe_threshold_mask(o.R_pre[idx], th, r.tol) & safe_threshold_mask(o.R_post[idx], th, r.tol)
+    assert np.array_equal(st[idx][safe], o.state[idx][safe])
+    assert safe.any()
+    nc = int(b.n_cand[0])
+    if (st == o.state).all() and nc == len(o.cand) and np.array_equal(_np(b.cand[0])[:nc], o.cand):
+        stepR = _np(b.step_R[0])[:nc]
+        safe_s = safe_threshold_mask(o.step_R, cfg.tau_joint, r.tol)
+        upto = nc if safe_s.all() else int(np.argmin(safe_s))
+        _assert_close(stepR[:upto], o.step_R[:upto], r.tol, "step R")
+        if upto == nc:
+            assert np.array_equal(_np(b.accepted[0])[:dev.P_post], o.accepted)
+            n = int(b.n_idx[0])
+            # pending order depends on R+ of the observation pages; compare
+            # the index set when those priorities are separated
+            pr = o.R_post[dev.tr.pending]
+            srt = np.sort(pr)
+            if len(srt) < 2 or np.all(np.diff(srt) > 2 * r.tol * srt[1:]):
+                assert np.array_equal(_np(b.idx[0])[:n], o.I)
+
+
+def test_gapped_positions():
+    """Non-contiguous absolute positions (a cache compacted earlier)."""
+    r = get_run("small", 5, gapped=True)
+    b, dev, o = r.buf, r.dev, r.orc
+    b.score_pre()
+    b.score_post()
+    torch.cuda.synchronize()
+    _assert_close(_np(b.R_pre[0])[:dev.P_pre], o.R_pre[:dev.P_pre], r.tol, "R-")
+    _assert_close(_np(b.R_post[0]), o.R_post, r.tol, "R+")
+
+
+def test_layer_mask():
+    r = get_run("small", 0)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    mask = [0, 1]
+    pre, post = None, None
+    from oracle_bridge import problems
+    pre, post = problems(r.tr, layer_mask=np.array(mask, np.uint8))
+    Rw, Hw = core.page_effects(post, "explicit")
+    R = torch.zeros(dev.P_post, device="cuda")
+    H = torch.full((cfg.M, cfg.Hq, dev.P_post), 7.0, device="cuda")
+    ck.commitkv_page_effects(b.shape, [dev.post()], [R], head_R_out=[H], layer_mask=mask, workspace=b.ws)
+    torch.cuda.synchronize()
+    _assert_close(_np(R), Rw, r.tol, "masked R")
+    _assert_close(_np(H), Hw, r.tol, "masked per-head R (unselected layers = 0)")
+
+
+def test_batched_trajectories_match_single():
+    """Three trajectories of different lengths in one launch sequence give
+    the same effects as the oracle for each."""
+    cfgs = [synth.small_config("b0", L_pre=300, L_obs=40), synth.small_config("b1", L_pre=700, L_obs=90),
+            synth.small_config("b2", L_pre=450, L_obs=64)]
+    trs = [synth.make_trajectory(c, 10 + i, traj=i) for i, c in enumerate(cfgs)]
+    devs = [DeviceTrajectory.upload(t) for t in trs]
+    buf = StepBuffers(cfgs[1], devs)
+    buf.score_pre()
+    buf.score_post()
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+    for t, d, Rm, Rp in zip(trs, devs, buf.R_pre, buf.R_post):
+        o = OracleStep(t, "explicit")
+        _assert_close(_np(Rm)[:d.P_pre], o.R_pre[:d.P_pre], 2e-2, "batched R-")
+        _assert_close(_np(Rp), o.R_post, 2e-2, "batched R+")
+
+
+def test_edge_cases():
+    """Empty page list, zero-length pages, a probe row that sees nothing, a
+    cache shorter than one tile."""
+    cfg = synth.small_config("edge", L_pre=40, L_obs=8, W=4, G=8, B=16, planted_frac=0.0,
+                             event_len=(4, 12))
+    tr = synth.make_trajectory(cfg, 0)
+    # a zero-length page and a probe row before every resident token
+    tr.page_len = tr.page_len.copy()
+    tr.page_len[0] = 0
+    dev = DeviceTrajectory.upload(tr)
+    qpos = dev.qpos_post.clone()
+    qpos[0] = -1
+    dev.qpos_post = qpos
+    buf = StepBuffers(cfg, [dev])
+    buf.score_post()
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+    post = core.Problem(synth.values_f64(tr.K, "bf16"), synth.values_f64(tr.V, "bf16"), tr.pos,
+                        synth.values_f64(tr.Q_post, "bf16"), _np(qpos), tr.page_start, tr.page_len)
+    Rw, _ = core.page_effects(post, "explicit")
+    _assert_close(_np(buf.R_post[0]), Rw, 2e-2, "edge R+")
+    assert float(buf.R_post[0][0]) == 0.0
+    # no pages at all
+    empty = ck.TrajTensors(dev.K, dev.V, dev.pos, dev.Q_post, dev.qpos_post,
+                           dev.page_start[:0], dev.page_len[:0])
+    R0 = torch.zeros(0, device="cuda")
+    ck.commitkv_page_effects(buf.shape, [empty], [R0], workspace=buf.ws)
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+
+
+def test_device_input_errors_are_reported():
+    """Inputs only the device can check: overlapping pages, a candidate id
+    out of range, a NaN fill score.  Each is reported in the workspace status
+    and the context stays usable."""
+    r = get_run("small", 0)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    bad_len = dev.page_len.clone()
+    bad_len[1] = bad_len[1] + 40  # overlaps page 2
+    t = ck.TrajTensors(dev.K, dev.V, dev.pos, dev.Q_post, dev.qpos_post, dev.page_start, bad_len)
+    ck.commitkv_page_effects(b.shape, [t], b.R_post, workspace=b.ws)
+    assert b.status() == ck.COMMITKV_ERR_DEVICE_INPUT
+    b.score_post()
+    cand = torch.tensor([dev.P_post + 5], dtype=torch.int32, device="cuda")
+    n_cand = torch.tensor([1], dtype=torch.int32, device="cuda")
+    ck.commitkv_joint_test(b.shape, [dev.post()], b.stats, [cand], n_cand, cfg.tau_joint, b.accepted,
+                           workspace=b.ws)
+    assert b.status() == ck.COMMITKV_ERR_DEVICE_INPUT
+    fill = dev.fill.clone()
+    fill[3] = float("nan")
+    ck.commitkv_compact(b.shape, [dev.post()], b.accepted, [dev.pending], b.R_post, [fill], cfg.B, cfg.B_N,
+                        cfg.pending_cap, b.idx, b.n_idx, workspace=b.ws)
+    assert b.status() == ck.COMMITKV_ERR_DEVICE_INPUT
+    # the context is still usable
+    b.score_post()
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+
+
+def test_bounded_wait_times_out():
+    """A grid barrier that can never fill ends by its time limit with
+    COMMITKV_ERR_TIMEOUT, and the context stays usable."""
+    r = get_run("small", 0)
+    b = r.buf
+    ck.commitkv_test_barrier_timeout(b.ws, 2)
+    assert b.status() == ck.COMMITKV_ERR_TIMEOUT
+    b.score_post()
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
