@@ -50,6 +50,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default="qwen3_8b_32k")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling cases)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -152,6 +153,17 @@ def oracle_sample(cfg, tr, budget_s: float):
 # ----------------------------------------------------------------------------
 
 
+def config_of(args):
+    import dataclasses
+
+    from paper_2608_07855_gb300 import synth
+
+    cfg = synth.CONFIGS[args.config]
+    if args.layers:
+        cfg = dataclasses.replace(cfg, name=f"{cfg.name}_L{args.layers}", M=args.layers)
+    return cfg
+
+
 def algorithmic(cfg):
     """Scoring roofline terms per token: K and V read once (bytes) and
     QK^T + PV once (flops), summed over layers and KV heads."""
@@ -169,7 +181,7 @@ def run_ours(args, rank, world, local):
     from paper_2608_07855_gb300.workload import DeviceTrajectory, StepBuffers
 
     torch.cuda.set_device(local)
-    cfg = synth.CONFIGS[args.config]
+    cfg = config_of(args)
     n_traj = cfg.n_traj
     trs = [synth.make_trajectory(cfg, args.seed + 1000 * rank, traj=i) for i in range(n_traj)]
     devs = [DeviceTrajectory.upload(t) for t in trs]
@@ -334,7 +346,7 @@ def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):
 def run_reference(args, rank, world):
     from paper_2608_07855_gb300 import synth
 
-    cfg = synth.CONFIGS[args.config]
+    cfg = config_of(args)
     if rank != 0:
         return None
     tr = synth.make_trajectory(cfg, args.seed, traj=0)
