@@ -3,7 +3,10 @@
 #include <math.h>
 #include <string.h>
 
+#include <stdlib.h>
+
 #include "ckv_internal.cuh"
+#include "score_tc.cuh"
 
 namespace ckv {
 int simt_rows_per_block();
@@ -100,6 +103,56 @@ int chunk_len_for(int n_traj, const commitkv_traj *tr) {
 
 int cdiv(int a, int b) { return (a + b - 1) / b; }
 
+// ---- tensor-core scoring path (bf16, head_dim 128)
+int tc_chunk_len(int n_traj, const commitkv_traj *tr) {
+  int smax = 0;
+  for (int t = 0; t < n_traj; ++t) smax = tr[t].S > smax ? tr[t].S : smax;
+  int c = (smax + 15) / 16;
+  if (c < 1024) c = 1024;
+  return (c + 127) / 128 * 128;
+}
+
+struct TcCounts {
+  int nchunk, nrt, nbitem;
+};
+
+TcCounts tc_counts(const commitkv_shape *s, const commitkv_traj &x, int CL) {
+  TcCounts c;
+  int g = s->q_heads / s->kv_heads;
+  c.nchunk = cdiv(x.S, CL);
+  c.nrt = cdiv(g * x.W, tc::kRowsPerTile);
+  c.nbitem = cdiv(cdiv(x.S, 16) + x.P, tc::kSlotsPerItem);
+  return c;
+}
+
+bool env_force_simt() {
+  const char *e = getenv("COMMITKV_SCORING");
+  return e && (e[0] == 's' || e[0] == 'S');
+}
+
+bool tc_eligible(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
+  if (s->dtype != COMMITKV_BF16 || s->head_dim != 128 || env_force_simt()) return false;
+  for (int t = 0; t < n_traj; ++t) {
+    const commitkv_traj &x = tr[t];
+    if (x.S == 0 || x.W == 0 || x.P == 0) continue;
+    if (((uintptr_t)x.k | (uintptr_t)x.v | (uintptr_t)x.q) % 16) return false;
+    if ((x.stride_tok * 2) % 16 || (x.stride_head * 2) % 16 || (x.stride_layer * 2) % 16) return false;
+    if (x.stride_head == 0 || x.stride_layer == 0) return false;
+  }
+  return true;
+}
+
+size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
+  int CL = tc_chunk_len(n_traj, tr);
+  size_t items = 0, slots = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    TcCounts c = tc_counts(s, tr[t], CL);
+    items += (size_t)s->layers * s->kv_heads * c.nchunk * c.nrt;
+    slots += align_up((size_t)(tr[t].P + 1) * 4);
+  }
+  return align_up(items * tc::kRowsPerTile * 132 * 4) + slots;
+}
+
 // Region sizes of each call (bytes after the 256-byte header).
 size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, int n_layers) {
   int CL = chunk_len_for(n_traj, tr), RB = simt_rows_per_block(), d = s->head_dim;
@@ -110,7 +163,12 @@ size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
     units += (size_t)n_layers * s->kv_heads * cdiv(tr[t].S, CL) * cdiv(rows, RB);
     stats += align_up((size_t)s->layers * s->q_heads * tr[t].W * (d + 4) * 4);
   }
-  return align_up(units * RB * (d + 4) * 4) + stats;
+  size_t scratch = align_up(units * RB * (d + 4) * 4);
+  if (s->head_dim == 128) {
+    size_t tcb = tc_score_bytes(s, n_traj, tr);
+    if (tcb > scratch) scratch = tcb;
+  }
+  return scratch + stats;
 }
 
 size_t joint_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, int n_layers) {
@@ -236,12 +294,17 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
     units += (size_t)nl * shape->kv_heads * L.nchunk[t] * L.nrb[t];
   }
   float *partials = reinterpret_cast<float *>(base);
-  char *sbase = base + align_up(units * RB * (d + 4) * 4);
-  // (the layout is computed for every layer; a mask only uses a prefix)
+  // scratch (either path's partials) first, then the stats of trajectories
+  // without stats_out; the layout is computed for every layer
   size_t full_units = 0;
   for (int t = 0; t < n_traj; ++t)
     full_units += (size_t)shape->layers * shape->kv_heads * L.nchunk[t] * L.nrb[t];
-  sbase = base + align_up(full_units * RB * (d + 4) * 4);
+  size_t scratch = align_up(full_units * RB * (d + 4) * 4);
+  if (shape->head_dim == 128) {
+    size_t tcb = tc_score_bytes(shape, n_traj, trajs);
+    if (tcb > scratch) scratch = tcb;
+  }
+  char *sbase = base + scratch;
   for (int t = 0; t < n_traj; ++t) {
     size_t sb = align_up((size_t)shape->layers * shape->q_heads * trajs[t].W * (d + 4) * 4);
     L.stats[t] = (stats_out && stats_out[t]) ? stats_out[t] : reinterpret_cast<float *>(sbase);
@@ -257,7 +320,68 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
     if (e != cudaSuccess) return cuda_status(e);
   }
   WsHeader *hdr = static_cast<WsHeader *>(workspace);
-  return cuda_status(launch_score_simt(L, partials, hdr, stream));
+  if (!tc_eligible(shape, n_traj, trajs)) return cuda_status(launch_score_simt(L, partials, hdr, stream));
+  // tensor-core path: trajectories in launches of up to tc::kMaxTc
+  static thread_local tc::TcLaunch T;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_status(e);
+  int CLt = tc_chunk_len(n_traj, trajs);
+  float *tc_partials = reinterpret_cast<float *>(base);
+  size_t items_all = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    TcCounts c = tc_counts(shape, trajs[t], CLt);
+    items_all += (size_t)shape->layers * shape->kv_heads * c.nchunk * c.nrt;
+  }
+  char *slot_base = base + align_up(items_all * tc::kRowsPerTile * 132 * 4);
+  for (int b0 = 0; b0 < n_traj; b0 += tc::kMaxTc) {
+    int nb = n_traj - b0 < tc::kMaxTc ? n_traj - b0 : tc::kMaxTc;
+    memset(&T, 0, sizeof T);
+    T.n_traj = nb;
+    T.M = shape->layers;
+    T.H = shape->kv_heads;
+    T.Hq = shape->q_heads;
+    T.g = L.batch.g;
+    T.n_layers = nl;
+    T.chunk_len = CLt;
+    T.slots_per_item = tc::kSlotsPerItem;
+    T.scale_log2 = L.batch.scale_log2;
+    T.partials = tc_partials;
+    memcpy(T.layer_ids, L.batch.layer_ids, sizeof T.layer_ids);
+    for (int i = 0; i < nb; ++i) {
+      int t = b0 + i;
+      const commitkv_traj &x = trajs[t];
+      TcCounts c = tc_counts(shape, x, CLt);
+      tc::TcTraj &tt = T.t[i];
+      tt.pos = x.pos;
+      tt.qpos = x.q_pos;
+      tt.ps = x.page_start;
+      tt.pl = x.page_len;
+      tt.slot_off = reinterpret_cast<int32_t *>(slot_base);
+      slot_base += align_up((size_t)(x.P + 1) * 4);
+      tt.stats = L.stats[t];
+      tt.R = L.R[t];
+      tt.headR = L.headR[t];
+      tt.S = x.S;
+      tt.W = x.W;
+      tt.P = x.P;
+      tt.nchunk = c.nchunk;
+      tt.nrt = c.nrt;
+      tt.nbitem = c.nbitem;
+      bool active = x.S > 0 && x.W > 0;
+      int ia = active ? nl * shape->kv_heads * c.nchunk * c.nrt : 0;
+      int ib = active && x.P > 0 ? nl * shape->kv_heads * c.nbitem * c.nrt : 0;
+      T.item_off_a[i + 1] = T.item_off_a[i] + ia;
+      T.item_off_b[i + 1] = T.item_off_b[i] + ib;
+      T.row_off[i + 1] = T.row_off[i] + (active ? nl * shape->kv_heads * L.batch.g * x.W : 0);
+      if (active && !tc::build_maps(T.maps[i], L.batch.t[t], shape->layers, shape->kv_heads, shape->q_heads))
+        return COMMITKV_ERR_CUDA;
+    }
+    e = tc::launch_score_tc(T, hdr, stream, sms);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return COMMITKV_OK;
 }
 
 commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float *const *R_pre,

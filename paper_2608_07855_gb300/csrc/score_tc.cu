@@ -1,0 +1,978 @@
+// Page deletion effects (Section 3.2, Eq. 6-8) on the 5th-generation tensor
+// cores: bf16 K/V/Q, head_dim 128, fp32 accumulation in tensor memory.
+//
+//   pass A   persistent, warp-specialised flash forward over 128-token tiles
+//            of a token chunk: S = Q K^T (tcgen05, TMEM), online softmax in
+//            base 2 with a lazy max (O in TMEM is rescaled only when the row
+//            max grows by more than 2^8), O += P V (tcgen05); writes the
+//            chunk's (max, sum, count, O) per probe row.
+//   combine  merges a slice's chunk partials into the row stats
+//            (m, l, n, o) of the whole cache.
+//   slots    per trajectory, the prefix count of 16-token slots per page.
+//   pass B   persistent, over tiles of 8 slots: every page is loaded as
+//            16-row TMA boxes into slots of its own, so one page's columns
+//            never share a 16-wide MMA k-block with another page.
+//            S = Q K_slots^T; e = exp(s - m) on the page's visible tokens;
+//            U_E = sum_{i in E} e_i v_i by per-slot MMAs accumulating into
+//            one of two 128-column TMEM accumulators; a separate epilogue
+//            warpgroup reduces U_E to
+//              r = ||U_E - S_E o|| / ((l - S_E) ||o||)      (Eq. 6 with a = e / l)
+//            and max-reduces r over rows into R[E] (Eq. 7).
+// Every mbarrier wait is bounded (1 s); on expiry the kernel records
+// COMMITKV_ERR_TIMEOUT and all warps leave their loops.
+#include <cudaTypedefs.h>
+
+#include "ckv_internal.cuh"
+#include "sm103.cuh"
+#include "score_tc.cuh"
+
+namespace ckv {
+namespace tc {
+namespace {
+
+using namespace ckv::sm103;
+
+constexpr int D = 128;
+constexpr int BM = 128;  // probe rows per tile (MMA M)
+constexpr int BT = 128;  // KV rows per tile (MMA N of Q K^T, K of P V)
+constexpr int NST = 2;   // K/V pipeline stages
+constexpr int SLOT = 16;
+constexpr int SLOTS = BT / SLOT;  // slots per pass-B tile
+constexpr int NFIFO = 8;          // page-sum FIFO depth (>= SLOTS)
+constexpr uint64_t kWait = 1000000000ull;
+constexpr float kLazy = 8.0f;     // rescale O when the max grows by > 2^8
+
+constexpr uint32_t kTileBytes = BT * D * 2;  // 32 KB (two 16 KB halves)
+constexpr uint32_t kHalf = kTileBytes / 2;
+
+// ----------------------------------------------------------------- helpers
+__device__ __forceinline__ int traj_of(const int32_t *off, int n, int item) {
+  int t = 0;
+  while (t + 1 < n && item >= off[t + 1]) ++t;
+  return t;
+}
+
+__device__ __forceinline__ void tma4(void *dst, const CUtensorMap *m, int x, int tok, int h, int l,
+                                     uint64_t *bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(tok), "r"(h), "r"(l), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
+}
+
+__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+
+// K-major operand tile (rows x 128 elements, two 64-element halves): the
+// descriptor of the 16-element k-step `ks`.
+__device__ __forceinline__ uint64_t desc_kmajor(const uint8_t *tile, int ks) {
+  return smem_desc(smem_addr(tile) + (ks >> 2) * kHalf + (ks & 3) * 32, 16, 1024, kSwizzle128B);
+}
+// MN-major B operand (V rows = k, 128 channels = n): k-step of 16 rows.
+__device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int ks) {
+  return smem_desc(smem_addr(tile) + ks * 2048, kHalf, 1024, kSwizzle128B);
+}
+
+// ============================================================== pass A
+// TMEM columns: S/P buffers at 0 and 128 (after the softmax reads a 32-column
+// chunk of S it overwrites the same columns with 16 columns of P_hi and 16
+// of P_lo), O at 256.
+struct SmemA {
+  alignas(1024) uint8_t q[kTileBytes];
+  alignas(1024) uint8_t k[NST][kTileBytes];
+  alignas(1024) uint8_t v[NST][kTileBytes];
+  int pos[2][BT];
+  uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full, pv_done,
+      o_full, o_empty, drain;
+  uint32_t tmem;
+  int abort_flag;
+};
+
+struct ItemA {
+  int t, l, kvh, rt, c, li;
+};
+
+__device__ __forceinline__ ItemA decode_a(const TcLaunch &L, int item) {
+  ItemA it;
+  it.t = traj_of(L.item_off_a, L.n_traj, item);
+  const TcTraj &tr = L.t[it.t];
+  int local = item - L.item_off_a[it.t];
+  it.rt = local % tr.nrt;
+  local /= tr.nrt;
+  it.c = local % tr.nchunk;
+  local /= tr.nchunk;
+  it.kvh = local % L.H;
+  it.li = local / L.H;
+  it.l = L.layer_ids[it.li];
+  return it;
+}
+
+// TMEM column of the 8 packed P columns (hi or lo) of k-step ks inside S/P buffer b.
+__device__ __forceinline__ uint32_t p_col(int b, int ks, int lo) {
+  return b * BT + 32 * (ks >> 1) + 8 * (ks & 1) + 16 * lo;
+}
+
+// Issues S[b] = Q K^T for one tile (8 k-steps over the 128 channels).
+__device__ __forceinline__ void issue_qk(uint32_t tm, const uint8_t *q, const uint8_t *k, int b) {
+  const uint32_t idesc = idesc_bf16_f32(BM, BT, 0, 0);
+#pragma unroll
+  for (int ks = 0; ks < D / 16; ++ks) mma_bf16(tm + b * BT, desc_kmajor(q, ks), desc_kmajor(k, ks), idesc, ks > 0);
+}
+
+// Issues D (+)= P[:, 16 ks .. 16 ks + 15] V[16 ks .. 16 ks + 15, :] with P as
+// the (hi, lo) pair in TMEM buffer b; `first` overwrites D.
+__device__ __forceinline__ void issue_pv_step(uint32_t tm, uint32_t d_col, const uint8_t *v, int b, int ks,
+                                              bool first) {
+  const uint32_t idesc = idesc_bf16_f32(BM, D, 0, 1);
+  uint64_t bd = desc_v(v, ks);
+  mma_bf16_ts(tm + d_col, tm + p_col(b, ks, 0), bd, idesc, first ? 0u : 1u);
+  mma_bf16_ts(tm + d_col, tm + p_col(b, ks, 1), bd, idesc, 1u);
+}
+
+__global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  SmemA &sm = *reinterpret_cast<SmemA *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n_items = L.item_off_a[L.n_traj];
+  volatile int *abort_flag = &sm.abort_flag;
+
+  if (threadIdx.x == 0) {
+    sm.abort_flag = 0;
+    mbar_init(&sm.q_full, 1);
+    mbar_init(&sm.q_empty, 1);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.v_full[s], 1);
+      mbar_init(&sm.kv_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.s_full[b], 1);
+      mbar_init(&sm.s_empty[b], 1);
+    }
+    mbar_init(&sm.p_full, 4);
+    mbar_init(&sm.pv_done, 1);
+    mbar_init(&sm.o_full, 1);
+    mbar_init(&sm.o_empty, 4);
+    mbar_init(&sm.drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = sm.tmem;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint64_t pol = policy_evict_normal();
+      uint32_t it = 0, n_local = 0;
+      for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++n_local) {
+        if (*abort_flag) break;
+        ItemA a = decode_a(L, item);
+        const TcTraj &tr = L.t[a.t];
+        const TcMaps &mp = L.maps[a.t];
+        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) break;
+        mbar_expect_tx(&sm.q_full, kTileBytes);
+        int qrow = (a.l * L.Hq + a.kvh * L.g) * tr.W + a.rt * BM;
+        tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+        tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
+        int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
+        bool stop = false;
+        for (int tok = t0; tok < t1; tok += BT, ++it) {
+          int s = it % NST;
+          if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
+            stop = true;
+            break;
+          }
+          mbar_expect_tx(&sm.k_full[s], kTileBytes);
+          tma4(sm.k[s], &mp.k, 0, tok, a.kvh, a.l, &sm.k_full[s], pol);
+          tma4(sm.k[s] + kHalf, &mp.k, 64, tok, a.kvh, a.l, &sm.k_full[s], pol);
+          mbar_expect_tx(&sm.v_full[s], kTileBytes);
+          tma4(sm.v[s], &mp.v, 0, tok, a.kvh, a.l, &sm.v_full[s], pol);
+          tma4(sm.v[s] + kHalf, &mp.v, 64, tok, a.kvh, a.l, &sm.v_full[s], pol);
+        }
+        if (stop) break;
+      }
+      if (*abort_flag) {
+        // let the copies already issued land before the CTA leaves
+        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
+          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
+          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
+        }
+        if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, n_local = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+        ItemA a = decode_a(L, item);
+        const TcTraj &tr = L.t[a.t];
+        int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
+        int ntile = (t1 - t0 + BT - 1) / BT;
+        if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
+        tc_fence_after();
+        auto qk = [&](uint32_t g) -> bool {
+          int s = g % NST, b = g & 1;
+          if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
+          if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
+          tc_fence_after();
+          issue_qk(tm, sm.q, sm.k[s], b);
+          mma_commit(&sm.s_full[b]);
+          return true;
+        };
+        if (ntile > 0) ok = qk(it);
+        // the O of the previous item must have been read out before P V overwrites it
+        if (ok && n_local > 0 && !mbar_wait(&sm.o_empty, (n_local - 1) & 1, kWait, abort_flag)) ok = false;
+        for (int j = 0; j < ntile && ok; ++j) {
+          uint32_t g = it + j;
+          if (j + 1 < ntile) {
+            ok = qk(g + 1);
+            if (!ok) break;
+          } else {
+            mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
+          }
+          int s = g % NST, b = g & 1;
+          if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
+              !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int ks = 0; ks < BT / 16; ++ks) issue_pv_step(tm, 2 * BT, sm.v[s], b, ks, j == 0 && ks == 0);
+          mma_commit(&sm.s_empty[b]);
+          mma_commit(&sm.kv_empty[s]);
+          mma_commit(&sm.pv_done);
+          if (j + 1 == ntile) mma_commit(&sm.o_full);
+        }
+        it += ntile;
+      }
+      if (*abort_flag) {
+        mma_commit(&sm.drain);  // every MMA issued by this thread has completed
+        mbar_wait_drain(&sm.drain, 0, kWait);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ softmax (warps 2..5)
+    const int wq = warp & 3;          // TMEM lane quarter of this warp
+    const int row = wq * 32 + lane;   // probe row within the tile
+    const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    uint32_t it = 0, n_local = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+      ItemA a = decode_a(L, item);
+      const TcTraj &tr = L.t[a.t];
+      int rows = L.g * tr.W;
+      int grow = a.rt * BM + row;  // row within the (layer, KV head) slice
+      bool valid_row = grow < rows;
+      int qp = valid_row ? tr.qpos[grow % tr.W] : -0x7fffffff;
+      int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
+      int ntile = (t1 - t0 + BT - 1) / BT;
+      float m_used = -INFINITY, m_true = -INFINITY, lsum = 0.0f;
+      int nvis = 0;
+      for (int j = 0; j < ntile && ok; ++j) {
+        uint32_t g = it + j;
+        int b = g & 1;
+        int tok0 = t0 + j * BT, nt = min(BT, t1 - tok0);
+        sm.pos[b][row] = row < nt ? tr.pos[tok0 + row] : 0x7fffffff;
+        named_sync(1, 128);
+        if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float x[BT];
+#pragma unroll
+        for (int c0 = 0; c0 < BT; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32(tm + lane_base + b * BT + c0, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) x[c0 + i] = __uint_as_float(r[i]);
+        }
+        float mt = -INFINITY;
+        int cnt = 0;
+#pragma unroll
+        for (int i = 0; i < BT; ++i) {
+          bool vis = i < nt && sm.pos[b][i] <= qp;
+          x[i] = vis ? x[i] * L.scale_log2 : -INFINITY;
+          mt = fmaxf(mt, x[i]);
+          cnt += vis;
+        }
+        nvis += cnt;
+        m_true = fmaxf(m_true, mt);
+        float m_new = fmaxf(m_used, mt);
+        bool rescale = m_new > m_used + kLazy;  // false while both are -inf
+        float alpha = (rescale && m_used != -INFINITY) ? exp2f(m_used - m_new) : 0.0f;
+        if (rescale) m_used = m_new;
+        // P V of the previous tile done: O is stable (phase g-1 of pv_done)
+        if (g > 0 && !mbar_wait(&sm.pv_done, (g - 1) & 1, kWait, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (j > 0 && __any_sync(0xffffffffu, rescale)) {
+          float f = rescale ? alpha : 1.0f;
+#pragma unroll
+          for (int c0 = 0; c0 < D; c0 += 32) {
+            uint32_t r[32];
+            tmem_ld32(tm + lane_base + 2 * BT + c0, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * f);
+            tmem_st32(tm + lane_base + 2 * BT + c0, r);
+          }
+          tmem_wait_st();
+        }
+        if (rescale) lsum *= alpha;
+        float ps = 0.0f;
+#pragma unroll
+        for (int c0 = 0; c0 < BT; c0 += 32) {
+          float p[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            p[i] = x[c0 + i] == -INFINITY ? 0.0f : exp2f(x[c0 + i] - m_used);
+            ps += p[i];
+          }
+          uint32_t pk[32];
+          split_pack32(p, pk);
+          tmem_st32(tm + lane_base + b * BT + c0, pk);
+        }
+        tmem_wait_st();
+        lsum += ps;
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.p_full);
+      }
+      if (!ok) break;
+      // item done: O complete after the last P V
+      if (!mbar_wait(&sm.o_full, n_local & 1, kWait, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float *dst = L.partials + ((int64_t)item * BM + row) * (D + 4);
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld32(tm + lane_base + 2 * BT + c0, r);
+        tmem_wait_ld();
+        if (valid_row) {
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            *reinterpret_cast<float4 *>(dst + 4 + c0 + i) =
+                make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]), __uint_as_float(r[i + 2]),
+                            __uint_as_float(r[i + 3]));
+        }
+      }
+      // (reference max of l and O, sum, visible count, true max)
+      if (valid_row) *reinterpret_cast<float4 *>(dst) = make_float4(m_used, lsum, (float)nvis, m_true);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.o_empty);
+      it += ntile;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tm, 512);
+  if (threadIdx.x == 0 && sm.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, 10);
+}
+
+// ============================================================== combine
+// One warp per probe row of the selected layers.
+__global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaunch L) {
+  int gw = (blockIdx.x * 256 + threadIdx.x) / 32, lane = threadIdx.x % 32;
+  int total = L.row_off[L.n_traj];
+  if (gw >= total) return;
+  int t = traj_of(L.row_off, L.n_traj, gw);
+  const TcTraj &tr = L.t[t];
+  int local = gw - L.row_off[t];
+  int rows = L.g * tr.W;
+  int row = local % rows;
+  local /= rows;
+  int kvh = local % L.H, li = local / L.H;
+  int l = L.layer_ids[li];
+  int rt = row / BM, rl = row % BM;
+  auto part = [&](int c) {
+    int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + c) * tr.nrt + rt;
+    return L.partials + ((int64_t)item * BM + rl) * (D + 4);
+  };
+  float m = -INFINITY;  // true row max over the chunks (base 2)
+  for (int c = 0; c < tr.nchunk; ++c) m = fmaxf(m, part(c)[3]);
+  float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+  float lsum = 0.0f, n = 0.0f;
+  for (int c = 0; c < tr.nchunk; ++c) {
+    const float *p = part(c);
+    n += p[2];
+    if (p[0] == -INFINITY) continue;
+    float a = exp2f(p[0] - m);
+    lsum = fmaf(p[1], a, lsum);
+    float4 v = *reinterpret_cast<const float4 *>(p + 4 + lane * 4);
+    o.x = fmaf(v.x, a, o.x);
+    o.y = fmaf(v.y, a, o.y);
+    o.z = fmaf(v.z, a, o.z);
+    o.w = fmaf(v.w, a, o.w);
+  }
+  float inv = lsum > 0.0f ? 1.0f / lsum : 0.0f;
+  int h = kvh * L.g + row / tr.W, w = row % tr.W;
+  float *dst = tr.stats + (((int64_t)l * L.Hq + h) * tr.W + w) * (D + 4);
+  if (lane == 0) *reinterpret_cast<float4 *>(dst) = make_float4(m == -INFINITY ? m : m * 0.69314718055994531f, lsum, n, 0.0f);
+  *reinterpret_cast<float4 *>(dst + 4 + lane * 4) = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
+}
+
+// ============================================================== slot offsets
+// slot_off[E] = sum over F < E of ceil(len_F / 16); slot_off[P] = total.
+// Also checks the page table (spans inside the cache, sorted, disjoint).
+__global__ void __launch_bounds__(1024) slots_kernel(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  const TcTraj &tr = L.t[blockIdx.x];
+  __shared__ int s_warp[32];
+  __shared__ int s_base;
+  if (threadIdx.x == 0) s_base = 0;
+  __syncthreads();
+  int lane = threadIdx.x % 32, wid = threadIdx.x / 32;
+  for (int c0 = 0; c0 < tr.P; c0 += 1024) {
+    int E = c0 + threadIdx.x;
+    int v = 0;
+    if (E < tr.P) {
+      int ps = tr.ps[E], pl = tr.pl[E];
+      bool bad = pl < 0 || ps < 0 || ps > tr.S - pl || (E > 0 && ps < tr.ps[E - 1] + tr.pl[E - 1]);
+      if (bad) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, E);
+      v = bad ? 0 : (pl + SLOT - 1) / SLOT;
+    }
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_warp[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+      int w = s_warp[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      s_warp[lane] = w;
+    }
+    __syncthreads();
+    int excl = s_base + (wid ? s_warp[wid - 1] : 0) + x - v;
+    if (E < tr.P) tr.slot_off[E] = excl;
+    __syncthreads();
+    if (threadIdx.x == 0) s_base += s_warp[31];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) tr.slot_off[tr.P] = s_base;
+}
+
+// ============================================================== pass B
+// TMEM columns: S/P buffers at 0 and 128 (as in pass A), page accumulators
+// U[0] at 256 and U[1] at 384.
+struct SlotMeta {
+  int tok0;   // first resident index of the slot
+  int nv;     // valid tokens in the slot (0 for an empty slot)
+  int po;     // page ordinal within the CTA's page stream (-1: empty slot)
+  int flags;  // bit 0: first slot of its page, bit 1: last slot of its page
+};
+
+struct SmemB {
+  alignas(1024) uint8_t q[kTileBytes];
+  alignas(1024) uint8_t k[NST][kTileBytes];
+  alignas(1024) uint8_t v[NST][kTileBytes];
+  SlotMeta meta[NST][SLOTS];
+  int page_of[NST][SLOTS];  // page id of each slot
+  int pos[2][BT];
+  float fifo_s[NFIFO][BM];  // per page: S_E of every row
+  int fifo_n[NFIFO][BM];    // per page: visible count of every row
+  int fifo_page[NFIFO];
+  uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full,
+      acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain;
+  uint32_t tmem;
+  int abort_flag;
+};
+
+struct ItemB {
+  int t, l, kvh, rt, k, li;
+  int E0, E1;        // pages [E0, E1)
+  int slot0, nslot;  // slots of those pages
+};
+
+__device__ __forceinline__ int lower_bound_i(const int32_t *a, int n, int key) {
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    int mid = (lo + hi) >> 1;
+    if (a[mid] < key) lo = mid + 1;
+    else hi = mid;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
+  ItemB b;
+  b.t = traj_of(L.item_off_b, L.n_traj, item);
+  const TcTraj &tr = L.t[b.t];
+  int local = item - L.item_off_b[b.t];
+  b.rt = local % tr.nrt;
+  local /= tr.nrt;
+  b.k = local % tr.nbitem;
+  local /= tr.nbitem;
+  b.kvh = local % L.H;
+  b.li = local / L.H;
+  b.l = L.layer_ids[b.li];
+  int lo = b.k * L.slots_per_item, hi = lo + L.slots_per_item;
+  b.E0 = lower_bound_i(tr.slot_off, tr.P, lo);
+  b.E1 = lower_bound_i(tr.slot_off, tr.P, hi);
+  b.slot0 = b.E0 < tr.P ? tr.slot_off[b.E0] : 0;
+  b.nslot = (b.E1 > b.E0) ? tr.slot_off[b.E1] - b.slot0 : 0;
+  return b;
+}
+
+__device__ __forceinline__ bool has_slots(const TcTraj &tr, int E) { return tr.slot_off[E + 1] > tr.slot_off[E]; }
+
+__global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  SmemB &sm = *reinterpret_cast<SmemB *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int n_items = L.item_off_b[L.n_traj];
+  volatile int *abort_flag = &sm.abort_flag;
+
+  if (threadIdx.x == 0) {
+    sm.abort_flag = 0;
+    mbar_init(&sm.q_full, 1);
+    mbar_init(&sm.q_empty, 1);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.v_full[s], 1);
+      mbar_init(&sm.kv_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.s_full[b], 1);
+      mbar_init(&sm.s_empty[b], 1);
+      mbar_init(&sm.acc_full[b], 1);
+      mbar_init(&sm.acc_empty[b], 4);
+    }
+    mbar_init(&sm.p_full, 4);
+    for (int f = 0; f < NFIFO; ++f) {
+      mbar_init(&sm.fifo_full[f], 4);
+      mbar_init(&sm.fifo_empty[f], 4);
+    }
+    mbar_init(&sm.drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = sm.tmem;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint64_t pol = policy_evict_first();
+      uint32_t it = 0, n_local = 0;
+      int po = 0;  // page ordinal
+      bool stop = false;
+      for (int item = blockIdx.x; item < n_items && !stop && !*abort_flag; item += gridDim.x) {
+        ItemB bi = decode_b(L, item);
+        if (bi.nslot == 0) continue;
+        const TcTraj &tr = L.t[bi.t];
+        const TcMaps &mp = L.maps[bi.t];
+        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) break;
+        mbar_expect_tx(&sm.q_full, kTileBytes);
+        int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
+        tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+        tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
+        ++n_local;
+        // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
+        int E = bi.E0, sub = 0;
+        while (E < bi.E1 && !has_slots(tr, E)) ++E;
+        int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+        for (int j = 0; j < ntile; ++j, ++it) {
+          int s = it % NST;
+          if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
+            stop = true;
+            break;
+          }
+          uint32_t bytes = 0;
+          for (int q = 0; q < SLOTS; ++q) {
+            SlotMeta mt;
+            if (E < bi.E1) {
+              int pl = tr.pl[E];
+              mt.tok0 = tr.ps[E] + sub * SLOT;
+              mt.nv = min(SLOT, pl - sub * SLOT);
+              mt.po = po;
+              mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
+              sm.page_of[s][q] = E;
+              bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
+              if (++sub * SLOT >= pl) {
+                sub = 0;
+                ++po;
+                ++E;
+                while (E < bi.E1 && !has_slots(tr, E)) ++E;
+              }
+            } else {
+              mt.tok0 = 0;
+              mt.nv = 0;
+              mt.po = -1;
+              mt.flags = 0;
+              sm.page_of[s][q] = -1;
+            }
+            sm.meta[s][q] = mt;
+          }
+          // the slot table is written before the arrivals that publish it
+          mbar_expect_tx(&sm.k_full[s], bytes);
+          mbar_expect_tx(&sm.v_full[s], bytes);
+          for (int q = 0; q < SLOTS; ++q) {
+            const SlotMeta &mt = sm.meta[s][q];
+            if (mt.po < 0) continue;
+            uint8_t *kd = sm.k[s] + q * SLOT * 128;
+            uint8_t *vd = sm.v[s] + q * SLOT * 128;
+            tma4(kd, &mp.kb, 0, mt.tok0, bi.kvh, bi.l, &sm.k_full[s], pol);
+            tma4(kd + kHalf, &mp.kb, 64, mt.tok0, bi.kvh, bi.l, &sm.k_full[s], pol);
+            tma4(vd, &mp.vb, 0, mt.tok0, bi.kvh, bi.l, &sm.v_full[s], pol);
+            tma4(vd + kHalf, &mp.vb, 64, mt.tok0, bi.kvh, bi.l, &sm.v_full[s], pol);
+          }
+        }
+      }
+      if (*abort_flag) {
+        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
+          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
+          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
+        }
+        if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, n_local = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        ItemB bi = decode_b(L, item);
+        if (bi.nslot == 0) continue;
+        int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+        if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
+        ++n_local;
+        tc_fence_after();
+        auto qk = [&](uint32_t g) -> bool {
+          int s = g % NST, b = g & 1;
+          if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
+          if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
+          tc_fence_after();
+          issue_qk(tm, sm.q, sm.k[s], b);
+          mma_commit(&sm.s_full[b]);
+          return true;
+        };
+        ok = qk(it);
+        for (int j = 0; j < ntile && ok; ++j) {
+          uint32_t g = it + j;
+          if (j + 1 < ntile) {
+            ok = qk(g + 1);
+            if (!ok) break;
+          } else {
+            mma_commit(&sm.q_empty);
+          }
+          int s = g % NST, b = g & 1;
+          if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
+              !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          for (int q = 0; q < SLOTS && ok; ++q) {
+            SlotMeta mt = sm.meta[s][q];
+            if (mt.po < 0) continue;
+            int a = mt.po & 1;
+            if ((mt.flags & 1) && mt.po >= 2) {
+              if (!mbar_wait(&sm.acc_empty[a], ((mt.po >> 1) - 1) & 1, kWait, abort_flag)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+            }
+            issue_pv_step(tm, 2 * BT + a * D, sm.v[s], b, q, (mt.flags & 1) != 0);
+            if (mt.flags & 2) mma_commit(&sm.acc_full[a]);
+          }
+          mma_commit(&sm.s_empty[b]);
+          mma_commit(&sm.kv_empty[s]);
+        }
+        it += ntile;
+      }
+      if (*abort_flag) {
+        mma_commit(&sm.drain);
+        mbar_wait_drain(&sm.drain, 0, kWait);
+      }
+    }
+  } else if (warp < 6) {
+    // ------------------------------------------------------------ softmax (warps 2..5)
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    uint32_t it = 0;
+    int po_seen = 0;
+    float S_cur = 0.0f;
+    int n_cur = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      ItemB bi = decode_b(L, item);
+      if (bi.nslot == 0) continue;
+      const TcTraj &tr = L.t[bi.t];
+      int rows = L.g * tr.W;
+      int grow = bi.rt * BM + row;
+      bool valid_row = grow < rows;
+      int qp = -0x7fffffff;
+      float m2 = -INFINITY;
+      if (valid_row) {
+        int h = bi.kvh * L.g + grow / tr.W, w = grow % tr.W;
+        qp = tr.qpos[w];
+        float mn = tr.stats[(((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4)];
+        m2 = mn == -INFINITY ? mn : mn * 1.4426950408889634f;
+      }
+      int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+      for (int j = 0; j < ntile && ok; ++j) {
+        uint32_t g = it + j;
+        int s = g % NST, b = g & 1;
+        // the slot table of this stage is published with its K copies
+        if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) {
+          ok = false;
+          break;
+        }
+        {
+          const SlotMeta mt = sm.meta[s][row / SLOT];
+          int i = row % SLOT;
+          sm.pos[b][row] = i < mt.nv ? tr.pos[mt.tok0 + i] : 0x7fffffff;
+        }
+        named_sync(1, 128);
+        if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        // e = exp(s - m) on the visible page tokens; fp32 slot sums; P as the
+        // (hi, lo) bf16 pair written over the S columns just read
+        float slot_s[SLOTS];
+        int slot_n[SLOTS];
+#pragma unroll
+        for (int c0 = 0; c0 < BT; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32(tm + lane_base + b * BT + c0, r);
+          tmem_wait_ld();
+          float e[32];
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            float ss = 0.0f;
+            int nn = 0;
+#pragma unroll
+            for (int i = 0; i < SLOT; ++i) {
+              int c = c0 + h2 * SLOT + i;
+              bool vis = valid_row && sm.pos[b][c] <= qp;
+              float v = vis ? exp2f(__uint_as_float(r[h2 * SLOT + i]) * L.scale_log2 - m2) : 0.0f;
+              e[h2 * SLOT + i] = v;
+              ss += v;
+              nn += vis;
+            }
+            slot_s[(c0 >> 4) + h2] = ss;
+            slot_n[(c0 >> 4) + h2] = nn;
+          }
+          uint32_t pk[32];
+          split_pack32(e, pk);
+          tmem_st32(tm + lane_base + b * BT + c0, pk);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.p_full);
+        // page sums: walk the slots in order, hand finished pages to the epilogue
+#pragma unroll
+        for (int q = 0; q < SLOTS; ++q) {
+          const SlotMeta mt = sm.meta[s][q];
+          if (mt.po < 0 || !ok) continue;
+          if (mt.flags & 1) {
+            S_cur = 0.0f;
+            n_cur = 0;
+          }
+          S_cur += slot_s[q];
+          n_cur += slot_n[q];
+          if (mt.flags & 2) {
+            int f = po_seen % NFIFO;
+            if (po_seen >= NFIFO &&
+                !mbar_wait(&sm.fifo_empty[f], ((po_seen / NFIFO) - 1) & 1, kWait, abort_flag)) {
+              ok = false;
+              continue;
+            }
+            sm.fifo_s[f][row] = S_cur;
+            sm.fifo_n[f][row] = n_cur;
+            if (row == 0) sm.fifo_page[f] = sm.page_of[s][q];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.fifo_full[f]);
+            ++po_seen;
+          }
+        }
+      }
+      it += ntile;
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 6..9)
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    int po = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      ItemB bi = decode_b(L, item);
+      if (bi.nslot == 0) continue;
+      const TcTraj &tr = L.t[bi.t];
+      int rows = L.g * tr.W;
+      int grow = bi.rt * BM + row;
+      bool valid_row = grow < rows;
+      int h = bi.kvh * L.g + (valid_row ? grow / tr.W : 0), w = valid_row ? grow % tr.W : 0;
+      float o[D];
+      float lsum = 0.0f, onorm = 0.0f;
+      int nvis = 0;
+      if (valid_row) {
+        const float *st = tr.stats + (((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4);
+        float4 hd = *reinterpret_cast<const float4 *>(st);
+        lsum = hd.y;
+        nvis = (int)hd.z;
+        float ss = 0.0f;
+#pragma unroll
+        for (int c = 0; c < D; c += 4) {
+          float4 v = *reinterpret_cast<const float4 *>(st + 4 + c);
+          o[c] = v.x;
+          o[c + 1] = v.y;
+          o[c + 2] = v.z;
+          o[c + 3] = v.w;
+          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+        onorm = sqrtf(ss);
+      } else {
+#pragma unroll
+        for (int c = 0; c < D; ++c) o[c] = 0.0f;
+      }
+      int npages = 0;
+      for (int E = bi.E0; E < bi.E1; ++E) npages += has_slots(tr, E);
+      for (int k = 0; k < npages && ok; ++k, ++po) {
+        int a = po & 1, f = po % NFIFO;
+        if (!mbar_wait(&sm.fifo_full[f], (po / NFIFO) & 1, kWait, abort_flag) ||
+            !mbar_wait(&sm.acc_full[a], (po >> 1) & 1, kWait, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float S_E = sm.fifo_s[f][row];
+        int n_E = sm.fifo_n[f][row];
+        int E = sm.fifo_page[f];
+        float num2 = 0.0f;
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32(tm + lane_base + 2 * BT + a * D + c0, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float dlt = fmaf(-S_E, o[c0 + i], __uint_as_float(r[i]));
+            num2 = fmaf(dlt, dlt, num2);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&sm.acc_empty[a]);
+          mbar_arrive(&sm.fifo_empty[f]);
+        }
+        float r = valid_row ? effect_value(n_E, nvis, S_E, lsum, num2, onorm) : 0.0f;
+        if (valid_row && tr.headR) atomic_max_nonneg(tr.headR + ((int64_t)bi.l * L.Hq + h) * tr.P + E, r);
+        float rm = r;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, off));
+        if (lane == 0) atomic_max_nonneg(tr.R + E, rm);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tm, 512);
+  if (threadIdx.x == 0 && sm.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, 11);
+}
+
+// ============================================================== host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+bool map_q(CUtensorMap *m, const void *q, uint64_t rows) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)D, rows};
+  cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  cuuint32_t box[2] = {64, BM};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(q), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool map_kv(CUtensorMap *m, const void *base, int S, int H, int M, int64_t st, int64_t sh, int64_t sl,
+            int box_rows) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)(S > 0 ? S : 1), (cuuint64_t)H, (cuuint64_t)M};
+  cuuint64_t strides[3] = {(cuuint64_t)st * 2, (cuuint64_t)sh * 2, (cuuint64_t)sl * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+size_t smem_a() { return sizeof(SmemA) + 1024; }
+size_t smem_b() { return sizeof(SmemB) + 1024; }
+
+bool build_maps(TcMaps &mp, const TrajDev &t, int M, int H, int Hq) {
+  uint64_t qrows = (uint64_t)M * Hq * (uint64_t)(t.W > 0 ? t.W : 1);
+  return map_q(&mp.q, t.q, qrows) && map_kv(&mp.k, t.k, t.S, H, M, t.st, t.sh, t.sl, BT) &&
+         map_kv(&mp.v, t.v, t.S, H, M, t.st, t.sh, t.sl, BT) &&
+         map_kv(&mp.kb, t.k, t.S, H, M, t.st, t.sh, t.sl, SLOT) &&
+         map_kv(&mp.vb, t.v, t.S, H, M, t.st, t.sh, t.sl, SLOT);
+}
+
+cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, int sm_count) {
+  cudaError_t e = cudaFuncSetAttribute(pass_a_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_a());
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(pass_b_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_b());
+  if (e != cudaSuccess) return e;
+  int na = L.item_off_a[L.n_traj];
+  if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 192, smem_a(), s>>>(L, hdr);
+  int rows = L.row_off[L.n_traj];
+  if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
+  slots_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
+  int nb = L.item_off_b[L.n_traj];
+  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 320, smem_b(), s>>>(L, hdr);
+  return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace ckv

@@ -1,0 +1,46 @@
+// Launch description of the tensor-core scoring path (score_tc.cu).
+#pragma once
+
+#include <cuda.h>
+
+#include "ckv_internal.cuh"
+
+namespace ckv {
+namespace tc {
+
+constexpr int kMaxTc = 16;          // trajectories per launch (tensor maps travel as parameters)
+constexpr int kRowsPerTile = 128;   // probe rows per MMA tile
+constexpr int kSlotsPerItem = 128;  // 16-token slots per pass-B work item
+
+struct TcMaps {
+  CUtensorMap q;       // Q as [M*Hq*W rows][128], box 64 x 128
+  CUtensorMap k, v;    // K, V as [M][H][S][128], box 64 x 128 x 1 x 1
+  CUtensorMap kb, vb;  // the same with 16-row boxes (page slots)
+};
+
+struct TcTraj {
+  const int32_t *pos, *qpos, *ps, *pl;
+  int32_t *slot_off;  // workspace [P + 1]
+  float *stats;       // [M][Hq][W][132]
+  float *R;           // [P]
+  float *headR;       // [M][Hq][P] or null
+  int S, W, P, nchunk, nrt, nbitem;
+};
+
+struct TcLaunch {
+  TcMaps maps[kMaxTc];
+  TcTraj t[kMaxTc];
+  int n_traj, M, H, Hq, g, n_layers, chunk_len, slots_per_item;
+  float scale_log2;
+  float *partials;  // [items_a][128][132]
+  int item_off_a[kMaxTc + 1], item_off_b[kMaxTc + 1], row_off[kMaxTc + 1];
+  uint8_t layer_ids[kMaxLayers];
+};
+
+size_t smem_a();
+size_t smem_b();
+bool build_maps(TcMaps &maps, const TrajDev &t, int M, int H, int Hq);
+cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count);
+
+}  // namespace tc
+}  // namespace ckv

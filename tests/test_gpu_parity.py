@@ -348,3 +348,24 @@ def test_bounded_wait_times_out():
     b.score_post()
     torch.cuda.synchronize()
     assert b.status() == ck.COMMITKV_OK
+
+
+@pytest.mark.parametrize("name,seed", [("small", 0), ("small_w40_g16", 2), ("small_long_pages", 4)])
+def test_scoring_paths_agree(name, seed, monkeypatch):
+    """The tensor-core scoring path (bf16, head_dim 128) and the CUDA-core
+    path give the same effects and stats within the bf16 tolerance."""
+    r = get_run(name, seed)
+    b, dev = r.buf, r.dev
+    out = {}
+    for path in ("tc", "simt"):
+        monkeypatch.setenv("COMMITKV_SCORING", path)
+        R = torch.zeros(dev.P_post, device="cuda")
+        st = torch.zeros_like(b.stats[0])
+        ck.commitkv_page_effects(b.shape, [dev.post()], [R], stats_out=[st], workspace=b.ws)
+        torch.cuda.synchronize()
+        assert b.status() == ck.COMMITKV_OK
+        out[path] = (_np(R), _np(st))
+    _assert_close(out["tc"][0], out["simt"][0], 2e-2, "R+ tc vs simt")
+    a, s_ = out["tc"][1].reshape(-1, r.cfg.d + 4), out["simt"][1].reshape(-1, r.cfg.d + 4)
+    assert np.array_equal(a[:, 2], s_[:, 2])
+    _assert_close(a[:, 0], s_[:, 0], 1e-5, "row max")
