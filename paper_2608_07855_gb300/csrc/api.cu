@@ -142,13 +142,24 @@ bool tc_eligible(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
   return true;
 }
 
+// Chunks per (layer, KV head) never exceed 16 nor ceil(S / 1024) for the
+// tensor-core path (ceil(S / 512) for the CUDA-core path), whatever S' <= S a
+// later call uses: the workspace bound below holds for smaller caches too.
+int tc_chunk_bound(int S) {
+  int c = cdiv(S, 1024);
+  return c < 16 ? c : 16;
+}
+int simt_chunk_bound(int S) {
+  int c = cdiv(S, 512);
+  return c < 16 ? c : 16;
+}
+
 size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
-  int CL = tc_chunk_len(n_traj, tr);
   size_t items = 0, slots = 0;
   for (int t = 0; t < n_traj; ++t) {
-    TcCounts c = tc_counts(s, tr[t], CL);
-    items += (size_t)s->layers * s->kv_heads * c.nchunk * c.nrt;
-    slots += align_up((size_t)(tr[t].P + 1) * 4);
+    TcCounts c = tc_counts(s, tr[t], tc_chunk_len(1, &tr[t]));
+    items += (size_t)s->layers * s->kv_heads * tc_chunk_bound(tr[t].S) * c.nrt;
+    slots += align_up((size_t)(tr[t].P + 1) * 4) + align_up((size_t)c.nbitem * 32) + kAlign;
   }
   return align_up(items * tc::kRowsPerTile * 132 * 4) + slots;
 }
@@ -158,9 +169,10 @@ size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
   int CL = chunk_len_for(n_traj, tr), RB = simt_rows_per_block(), d = s->head_dim;
   int g = s->q_heads / s->kv_heads;
   size_t units = 0, stats = 0;
+  (void)CL;
   for (int t = 0; t < n_traj; ++t) {
     int rows = g * tr[t].W;
-    units += (size_t)n_layers * s->kv_heads * cdiv(tr[t].S, CL) * cdiv(rows, RB);
+    units += (size_t)n_layers * s->kv_heads * simt_chunk_bound(tr[t].S) * cdiv(rows, RB);
     stats += align_up((size_t)s->layers * s->q_heads * tr[t].W * (d + 4) * 4);
   }
   size_t scratch = align_up(units * RB * (d + 4) * 4);
@@ -298,7 +310,7 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
   // without stats_out; the layout is computed for every layer
   size_t full_units = 0;
   for (int t = 0; t < n_traj; ++t)
-    full_units += (size_t)shape->layers * shape->kv_heads * L.nchunk[t] * L.nrb[t];
+    full_units += (size_t)shape->layers * shape->kv_heads * simt_chunk_bound(trajs[t].S) * L.nrb[t];
   size_t scratch = align_up(full_units * RB * (d + 4) * 4);
   if (shape->head_dim == 128) {
     size_t tcb = tc_score_bytes(shape, n_traj, trajs);
@@ -332,7 +344,7 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
   size_t items_all = 0;
   for (int t = 0; t < n_traj; ++t) {
     TcCounts c = tc_counts(shape, trajs[t], CLt);
-    items_all += (size_t)shape->layers * shape->kv_heads * c.nchunk * c.nrt;
+    items_all += (size_t)shape->layers * shape->kv_heads * tc_chunk_bound(trajs[t].S) * c.nrt;
   }
   char *slot_base = base + align_up(items_all * tc::kRowsPerTile * 132 * 4);
   for (int b0 = 0; b0 < n_traj; b0 += tc::kMaxTc) {
@@ -360,6 +372,10 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
       tt.pl = x.page_len;
       tt.slot_off = reinterpret_cast<int32_t *>(slot_base);
       slot_base += align_up((size_t)(x.P + 1) * 4);
+      tt.items = reinterpret_cast<int4 *>(slot_base);
+      slot_base += align_up((size_t)c.nbitem * 32);
+      tt.prep = reinterpret_cast<tc::TcPrep *>(slot_base);
+      slot_base += kAlign;
       tt.stats = L.stats[t];
       tt.R = L.R[t];
       tt.headR = L.headR[t];

@@ -61,7 +61,6 @@ __device__ __forceinline__ void tma4(void *dst, const CUtensorMap *m, int x, int
       : "memory");
 }
 
-__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
 
 // K-major operand tile (rows x 128 elements, two 64-element halves): the
 // descriptor of the 16-element k-step `ks`.
@@ -81,7 +80,7 @@ struct SmemA {
   alignas(1024) uint8_t q[kTileBytes];
   alignas(1024) uint8_t k[NST][kTileBytes];
   alignas(1024) uint8_t v[NST][kTileBytes];
-  int pos[2][BT];
+  int pos[4][BT];  // per softmax warp: positions of the current tile
   uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full, pv_done,
       o_full, o_empty, drain;
   uint32_t tmem;
@@ -273,6 +272,7 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
       int grow = a.rt * BM + row;  // row within the (layer, KV head) slice
       bool valid_row = grow < rows;
       int qp = valid_row ? tr.qpos[grow % tr.W] : -0x7fffffff;
+      const int vis_all = tr.prep->vis_all;
       int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
       int ntile = (t1 - t0 + BT - 1) / BT;
       float m_used = -INFINITY, m_true = -INFINITY, lsum = 0.0f;
@@ -281,31 +281,47 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         uint32_t g = it + j;
         int b = g & 1;
         int tok0 = t0 + j * BT, nt = min(BT, t1 - tok0);
-        sm.pos[b][row] = row < nt ? tr.pos[tok0 + row] : 0x7fffffff;
-        named_sync(1, 128);
+        // tiles inside the prefix every probe row sees need no position test
+        const bool full = tok0 + nt <= vis_all;
+        if (!full) {  // each warp keeps its own copy: no cross-warp barrier
+          __syncwarp();
+#pragma unroll
+          for (int i = lane; i < BT; i += 32) sm.pos[wq][i] = i < nt ? tr.pos[tok0 + i] : 0x7fffffff;
+          __syncwarp();
+        }
         if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
         float x[BT];
+        tmem_ld32f(tm + lane_base + b * BT + 0, x);
+        tmem_ld32f(tm + lane_base + b * BT + 32, x + 32);
+        tmem_ld32f(tm + lane_base + b * BT + 64, x + 64);
+        tmem_ld32f(tm + lane_base + b * BT + 96, x + 96);
+        tmem_wait_ld();
+        // raw scores: masked ones become -inf; max on the raw scale (scale > 0)
+        int cnt;
+        if (!(full && nt == BT && valid_row)) {
+          cnt = 0;
 #pragma unroll
-        for (int c0 = 0; c0 < BT; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32(tm + lane_base + b * BT + c0, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) x[c0 + i] = __uint_as_float(r[i]);
+          for (int i = 0; i < BT; ++i) {
+            bool vis = valid_row && i < nt && (full || sm.pos[wq][i] <= qp);
+            x[i] = vis ? x[i] : -INFINITY;
+            cnt += vis;
+          }
+        } else {
+          cnt = BT;
         }
-        float mt = -INFINITY;
-        int cnt = 0;
+        float mx[8];
 #pragma unroll
-        for (int i = 0; i < BT; ++i) {
-          bool vis = i < nt && sm.pos[b][i] <= qp;
-          x[i] = vis ? x[i] * L.scale_log2 : -INFINITY;
-          mt = fmaxf(mt, x[i]);
-          cnt += vis;
-        }
+        for (int k = 0; k < 8; ++k) mx[k] = x[k];
+#pragma unroll
+        for (int i = 8; i < BT; i += 8)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], x[i + k]);
+        float smax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        float mt = smax == -INFINITY ? smax : smax * L.scale_log2;
         nvis += cnt;
         m_true = fmaxf(m_true, mt);
         float m_new = fmaxf(m_used, mt);
@@ -332,17 +348,21 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
           tmem_wait_st();
         }
         if (rescale) lsum *= alpha;
-        float ps = 0.0f;
+        const float neg_m = m_used == -INFINITY ? 0.0f : -m_used;
+#pragma unroll
+        for (int i = 0; i < BT; ++i) x[i] = fast_exp2(fmaf(x[i], L.scale_log2, neg_m));  // 2^-inf = 0
+        float pacc[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) pacc[k] = x[k];
+#pragma unroll
+        for (int i = 8; i < BT; i += 8)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) pacc[k] += x[i + k];
+        float ps = ((pacc[0] + pacc[1]) + (pacc[2] + pacc[3])) + ((pacc[4] + pacc[5]) + (pacc[6] + pacc[7]));
 #pragma unroll
         for (int c0 = 0; c0 < BT; c0 += 32) {
-          float p[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            p[i] = x[c0 + i] == -INFINITY ? 0.0f : exp2f(x[c0 + i] - m_used);
-            ps += p[i];
-          }
           uint32_t pk[32];
-          split_pack32(p, pk);
+          split_pack32(x + c0, pk);
           tmem_st32(tm + lane_base + b * BT + c0, pk);
         }
         tmem_wait_st();
@@ -428,10 +448,15 @@ __global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaun
   *reinterpret_cast<float4 *>(dst + 4 + lane * 4) = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
 }
 
-// ============================================================== slot offsets
-// slot_off[E] = sum over F < E of ceil(len_F / 16); slot_off[P] = total.
-// Also checks the page table (spans inside the cache, sorted, disjoint).
-__global__ void __launch_bounds__(1024) slots_kernel(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+// ============================================================== prep
+// Per trajectory, once per call:
+//   slot_off[E] = sum over F < E of ceil(len_F / 16), slot_off[P] = total
+//   (a page that fails the table checks gets no slot and an error is recorded);
+//   the pass-B work items: item k takes the pages whose first slot lies in
+//   [k * slots_per_item, (k + 1) * slots_per_item);
+//   vis_all = number of leading resident tokens visible to every probe row
+//   (positions increase, so this is a prefix).
+__global__ void __launch_bounds__(1024) prep_kernel(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   const TcTraj &tr = L.t[blockIdx.x];
   __shared__ int s_warp[32];
   __shared__ int s_base;
@@ -472,6 +497,41 @@ __global__ void __launch_bounds__(1024) slots_kernel(const __grid_constant__ TcL
     __syncthreads();
   }
   if (threadIdx.x == 0) tr.slot_off[tr.P] = s_base;
+  __syncthreads();
+  for (int k = threadIdx.x; k < tr.nbitem; k += 1024) {
+    int lo = k * L.slots_per_item, hi = lo + L.slots_per_item;
+    int a = 0, b = tr.P;
+    while (a < b) {
+      int mid = (a + b) >> 1;
+      if (tr.slot_off[mid] < lo) a = mid + 1;
+      else b = mid;
+    }
+    int E0 = a;
+    b = tr.P;
+    while (a < b) {
+      int mid = (a + b) >> 1;
+      if (tr.slot_off[mid] < hi) a = mid + 1;
+      else b = mid;
+    }
+    int E1 = a;
+    int slot0 = E0 < tr.P ? tr.slot_off[E0] : 0;
+    int nslot = E1 > E0 ? tr.slot_off[E1] - slot0 : 0;
+    int npages = 0;
+    for (int E = E0; E < E1; ++E) npages += tr.slot_off[E + 1] > tr.slot_off[E];
+    tr.items[2 * k] = make_int4(E0, E1, slot0, nslot);
+    tr.items[2 * k + 1] = make_int4(npages, 0, 0, 0);
+  }
+  if (threadIdx.x == 0) {
+    int qmin = 0x7fffffff;
+    for (int w = 0; w < tr.W; ++w) qmin = min(qmin, tr.qpos[w]);
+    int a = 0, b = tr.S;  // first token with pos > qmin
+    while (a < b) {
+      int mid = (a + b) >> 1;
+      if (tr.pos[mid] <= qmin) a = mid + 1;
+      else b = mid;
+    }
+    tr.prep->vis_all = a;
+  }
 }
 
 // ============================================================== pass B
@@ -490,12 +550,16 @@ struct SmemB {
   alignas(1024) uint8_t v[NST][kTileBytes];
   SlotMeta meta[NST][SLOTS];
   int page_of[NST][SLOTS];  // page id of each slot
-  int pos[2][BT];
+  int pos[4][BT];           // per softmax warp: positions of the current tile
+  int pg_start[kSlotsPerItem];  // the producer's copy of the item's page table
+  int pg_len[kSlotsPerItem];
+  int pg_slots[kSlotsPerItem];
+  float red[2][BM];         // per page parity: the upper channel half of ||U - S o||^2
   float fifo_s[NFIFO][BM];  // per page: S_E of every row
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
   uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full,
-      acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain;
+      acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], red_full[2], red_empty[2], drain;
   uint32_t tmem;
   int abort_flag;
 };
@@ -505,16 +569,6 @@ struct ItemB {
   int E0, E1;        // pages [E0, E1)
   int slot0, nslot;  // slots of those pages
 };
-
-__device__ __forceinline__ int lower_bound_i(const int32_t *a, int n, int key) {
-  int lo = 0, hi = n;
-  while (lo < hi) {
-    int mid = (lo + hi) >> 1;
-    if (a[mid] < key) lo = mid + 1;
-    else hi = mid;
-  }
-  return lo;
-}
 
 __device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
   ItemB b;
@@ -528,17 +582,17 @@ __device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
   b.kvh = local % L.H;
   b.li = local / L.H;
   b.l = L.layer_ids[b.li];
-  int lo = b.k * L.slots_per_item, hi = lo + L.slots_per_item;
-  b.E0 = lower_bound_i(tr.slot_off, tr.P, lo);
-  b.E1 = lower_bound_i(tr.slot_off, tr.P, hi);
-  b.slot0 = b.E0 < tr.P ? tr.slot_off[b.E0] : 0;
-  b.nslot = (b.E1 > b.E0) ? tr.slot_off[b.E1] - b.slot0 : 0;
+  int4 e = tr.items[2 * b.k];
+  b.E0 = e.x;
+  b.E1 = e.y;
+  b.slot0 = e.z;
+  b.nslot = e.w;
   return b;
 }
 
 __device__ __forceinline__ bool has_slots(const TcTraj &tr, int E) { return tr.slot_off[E + 1] > tr.slot_off[E]; }
 
-__global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+__global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   extern __shared__ uint8_t smem_raw[];
   SmemB &sm = *reinterpret_cast<SmemB *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -558,12 +612,14 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
       mbar_init(&sm.s_full[b], 1);
       mbar_init(&sm.s_empty[b], 1);
       mbar_init(&sm.acc_full[b], 1);
-      mbar_init(&sm.acc_empty[b], 4);
+      mbar_init(&sm.acc_empty[b], 8);
+      mbar_init(&sm.red_full[b], 4);
+      mbar_init(&sm.red_empty[b], 4);
     }
     mbar_init(&sm.p_full, 4);
     for (int f = 0; f < NFIFO; ++f) {
       mbar_init(&sm.fifo_full[f], 4);
-      mbar_init(&sm.fifo_empty[f], 4);
+      mbar_init(&sm.fifo_empty[f], 8);
     }
     mbar_init(&sm.drain, 1);
     fence_mbar_init();
@@ -579,80 +635,123 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      uint64_t pol = policy_evict_first();
-      uint32_t it = 0, n_local = 0;
-      int po = 0;  // page ordinal
-      bool stop = false;
-      for (int item = blockIdx.x; item < n_items && !stop && !*abort_flag; item += gridDim.x) {
-        ItemB bi = decode_b(L, item);
-        if (bi.nslot == 0) continue;
-        const TcTraj &tr = L.t[bi.t];
-        const TcMaps &mp = L.maps[bi.t];
-        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) break;
-        mbar_expect_tx(&sm.q_full, kTileBytes);
-        int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
-        tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
-        tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
-        ++n_local;
-        // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
-        int E = bi.E0, sub = 0;
-        while (E < bi.E1 && !has_slots(tr, E)) ++E;
-        int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-        for (int j = 0; j < ntile; ++j, ++it) {
-          int s = it % NST;
-          if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
-            stop = true;
-            break;
-          }
-          uint32_t bytes = 0;
-          for (int q = 0; q < SLOTS; ++q) {
-            SlotMeta mt;
-            if (E < bi.E1) {
-              int pl = tr.pl[E];
-              mt.tok0 = tr.ps[E] + sub * SLOT;
-              mt.nv = min(SLOT, pl - sub * SLOT);
-              mt.po = po;
-              mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
-              sm.page_of[s][q] = E;
-              bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
-              if (++sub * SLOT >= pl) {
-                sub = 0;
-                ++po;
-                ++E;
-                while (E < bi.E1 && !has_slots(tr, E)) ++E;
-              }
-            } else {
-              mt.tok0 = 0;
-              mt.nv = 0;
-              mt.po = -1;
-              mt.flags = 0;
-              sm.page_of[s][q] = -1;
+    // The whole warp copies each item's page table into shared memory; lane 0
+    // then walks the slots and issues the copies.
+    uint64_t pol = policy_evict_first();
+    uint32_t it = 0, n_local = 0;
+    int po = 0;  // page ordinal
+    bool stop = false;
+    for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
+      if (*abort_flag) break;
+      ItemB bi = decode_b(L, item);
+      if (bi.nslot == 0) continue;
+      const TcTraj &tr = L.t[bi.t];
+      const TcMaps &mp = L.maps[bi.t];
+      // pages of the item; zero-length pages take no slot, so there may be more
+      // pages than the copy holds: those are read from global memory
+      int np = bi.E1 - bi.E0;
+      for (int e = lane; e < min(np, kSlotsPerItem); e += 32) {
+        int E = bi.E0 + e;
+        sm.pg_start[e] = tr.ps[E];
+        sm.pg_len[e] = tr.pl[E];
+        sm.pg_slots[e] = tr.slot_off[E + 1] - tr.slot_off[E];
+      }
+      __syncwarp();
+      if (lane == 0) {
+        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) {
+          stop = true;
+        } else {
+          mbar_expect_tx(&sm.q_full, kTileBytes);
+          int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
+          tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+          tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
+          ++n_local;
+          // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
+          auto pslots = [&](int e) {
+            return e < kSlotsPerItem ? sm.pg_slots[e] : tr.slot_off[bi.E0 + e + 1] - tr.slot_off[bi.E0 + e];
+          };
+          int e = 0, sub = 0;
+          while (e < np && pslots(e) == 0) ++e;
+          int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+          for (int j = 0; j < ntile; ++j, ++it) {
+            int s = it % NST;
+            if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
+              stop = true;
+              break;
             }
-            sm.meta[s][q] = mt;
-          }
-          // the slot table is written before the arrivals that publish it
-          mbar_expect_tx(&sm.k_full[s], bytes);
-          mbar_expect_tx(&sm.v_full[s], bytes);
-          for (int q = 0; q < SLOTS; ++q) {
-            const SlotMeta &mt = sm.meta[s][q];
-            if (mt.po < 0) continue;
-            uint8_t *kd = sm.k[s] + q * SLOT * 128;
-            uint8_t *vd = sm.v[s] + q * SLOT * 128;
-            tma4(kd, &mp.kb, 0, mt.tok0, bi.kvh, bi.l, &sm.k_full[s], pol);
-            tma4(kd + kHalf, &mp.kb, 64, mt.tok0, bi.kvh, bi.l, &sm.k_full[s], pol);
-            tma4(vd, &mp.vb, 0, mt.tok0, bi.kvh, bi.l, &sm.v_full[s], pol);
-            tma4(vd + kHalf, &mp.vb, 64, mt.tok0, bi.kvh, bi.l, &sm.v_full[s], pol);
+            uint32_t bytes = 0;
+#pragma unroll
+            for (int q = 0; q < SLOTS; ++q) {
+              SlotMeta mt;
+              if (e < np) {
+                int pl = e < kSlotsPerItem ? sm.pg_len[e] : tr.pl[bi.E0 + e];
+                mt.tok0 = (e < kSlotsPerItem ? sm.pg_start[e] : tr.ps[bi.E0 + e]) + sub * SLOT;
+                mt.nv = min(SLOT, pl - sub * SLOT);
+                mt.po = po;
+                mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
+                sm.page_of[s][q] = bi.E0 + e;
+                bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
+                if (++sub * SLOT >= pl) {
+                  sub = 0;
+                  ++po;
+                  ++e;
+                  while (e < np && pslots(e) == 0) ++e;
+                }
+              } else {
+                mt.tok0 = 0;
+                mt.nv = 0;
+                mt.po = -1;
+                mt.flags = 0;
+                sm.page_of[s][q] = -1;
+              }
+              sm.meta[s][q] = mt;
+            }
+            // the slot table is written before the arrivals that publish it
+            mbar_expect_tx(&sm.k_full[s], bytes);
+            mbar_expect_tx(&sm.v_full[s], bytes);
+            // runs of slots whose rows are contiguous in memory (full pages
+            // of one event) travel as one box of 16, 32, 64 or 128 rows
+            int q = 0;
+            while (q < SLOTS) {
+              const SlotMeta m0 = sm.meta[s][q];
+              if (m0.po < 0) {
+                ++q;
+                continue;
+              }
+              int run = 1;
+              while (q + run < SLOTS && sm.meta[s][q + run].po >= 0 &&
+                     sm.meta[s][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s][q + run - 1].nv == SLOT)
+                ++run;
+              int done = 0;
+              while (done < run) {
+                int rem = run - done;
+                int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
+                if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
+                int tok = m0.tok0 + done * SLOT;
+                uint8_t *kd = sm.k[s] + (q + done) * SLOT * 128;
+                uint8_t *vd = sm.v[s] + (q + done) * SLOT * 128;
+                const CUtensorMap *km = lg == 3 ? &mp.k : &mp.kb[lg];
+                const CUtensorMap *vm = lg == 3 ? &mp.v : &mp.vb[lg];
+                tma4(kd, km, 0, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
+                tma4(kd + kHalf, km, 64, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
+                tma4(vd, vm, 0, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
+                tma4(vd + kHalf, vm, 64, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
+                done += 1 << lg;
+              }
+              q += run;
+            }
           }
         }
       }
-      if (*abort_flag) {
-        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
-          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
-          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
-        }
-        if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
+      stop = __shfl_sync(0xffffffffu, stop, 0);
+      __syncwarp();
+    }
+    if (lane == 0 && *abort_flag) {
+      for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
+        mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
+        mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
       }
+      if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -733,13 +832,15 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
       int grow = bi.rt * BM + row;
       bool valid_row = grow < rows;
       int qp = -0x7fffffff;
-      float m2 = -INFINITY;
+      // rows outside the slice, or rows that see nothing, get e = 0 everywhere
+      float neg_m2 = -INFINITY;
       if (valid_row) {
         int h = bi.kvh * L.g + grow / tr.W, w = grow % tr.W;
         qp = tr.qpos[w];
         float mn = tr.stats[(((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4)];
-        m2 = mn == -INFINITY ? mn : mn * 1.4426950408889634f;
+        if (mn != -INFINITY) neg_m2 = -mn * 1.4426950408889634f;
       }
+      const int vis_all = tr.prep->vis_all;
       int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
       for (int j = 0; j < ntile && ok; ++j) {
         uint32_t g = it + j;
@@ -749,12 +850,23 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
           ok = false;
           break;
         }
-        {
-          const SlotMeta mt = sm.meta[s][row / SLOT];
-          int i = row % SLOT;
-          sm.pos[b][row] = i < mt.nv ? tr.pos[mt.tok0 + i] : 0x7fffffff;
+        // slots inside the prefix every probe row sees need no position test
+        bool full = true;
+#pragma unroll
+        for (int q = 0; q < SLOTS; ++q) {
+          const SlotMeta mt = sm.meta[s][q];
+          full &= mt.po < 0 || mt.tok0 + mt.nv <= vis_all;
         }
-        named_sync(1, 128);
+        if (!full) {  // each warp keeps its own copy: no cross-warp barrier
+          __syncwarp();
+#pragma unroll
+          for (int c = lane; c < BT; c += 32) {
+            const SlotMeta mt = sm.meta[s][c / SLOT];
+            int i = c % SLOT;
+            sm.pos[wq][c] = i < mt.nv ? tr.pos[mt.tok0 + i] : 0x7fffffff;
+          }
+          __syncwarp();
+        }
         if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
           ok = false;
           break;
@@ -764,31 +876,49 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
         // (hi, lo) bf16 pair written over the S columns just read
         float slot_s[SLOTS];
         int slot_n[SLOTS];
+        // 32-column chunks, software-pipelined: the load of chunk c + 1 is in
+        // flight while chunk c is computed (scores in, probabilities out, in place)
+        float eb[2][32];
+        tmem_ld32f(tm + lane_base + b * BT, eb[0]);
+        tmem_wait_ld();
 #pragma unroll
-        for (int c0 = 0; c0 < BT; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32(tm + lane_base + b * BT + c0, r);
-          tmem_wait_ld();
-          float e[32];
+        for (int ch = 0; ch < BT / 32; ++ch) {
+          float *e = eb[ch & 1];
+          if (ch + 1 < BT / 32) tmem_ld32f(tm + lane_base + b * BT + 32 * (ch + 1), eb[(ch + 1) & 1]);
 #pragma unroll
           for (int h2 = 0; h2 < 2; ++h2) {
-            float ss = 0.0f;
-            int nn = 0;
+            const int q = 2 * ch + h2;
+            const int nv = sm.meta[s][q].nv;
+            float *es = e + h2 * SLOT;
+            int nn;
+            if (full && nv == SLOT) {
 #pragma unroll
-            for (int i = 0; i < SLOT; ++i) {
-              int c = c0 + h2 * SLOT + i;
-              bool vis = valid_row && sm.pos[b][c] <= qp;
-              float v = vis ? exp2f(__uint_as_float(r[h2 * SLOT + i]) * L.scale_log2 - m2) : 0.0f;
-              e[h2 * SLOT + i] = v;
-              ss += v;
-              nn += vis;
+              for (int i = 0; i < SLOT; ++i) es[i] = fast_exp2(fmaf(es[i], L.scale_log2, neg_m2));
+              nn = valid_row ? SLOT : 0;
+            } else {
+              nn = 0;
+#pragma unroll
+              for (int i = 0; i < SLOT; ++i) {
+                bool vis = i < nv && (full || sm.pos[wq][32 * ch + h2 * SLOT + i] <= qp);
+                es[i] = vis ? fast_exp2(fmaf(es[i], L.scale_log2, neg_m2)) : 0.0f;
+                nn += vis && valid_row;
+              }
             }
-            slot_s[(c0 >> 4) + h2] = ss;
-            slot_n[(c0 >> 4) + h2] = nn;
+            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+            for (int i = 0; i < SLOT; i += 4) {
+              a0 += es[i];
+              a1 += es[i + 1];
+              a2 += es[i + 2];
+              a3 += es[i + 3];
+            }
+            slot_s[q] = (a0 + a1) + (a2 + a3);
+            slot_n[q] = nn;
           }
           uint32_t pk[32];
           split_pack32(e, pk);
-          tmem_st32(tm + lane_base + b * BT + c0, pk);
+          tmem_st32(tm + lane_base + b * BT + 32 * ch, pk);
+          if (ch + 1 < BT / 32) tmem_wait_ld();
         }
         tmem_wait_st();
         tc_fence_before();
@@ -824,10 +954,14 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
       it += ntile;
     }
   } else {
-    // ------------------------------------------------------------ epilogue (warps 6..9)
+    // ------------------------------------------------------------ epilogue (warps 6..13)
+    // Two warpgroups split the 128 channels; each thread owns one row and 64
+    // channels of that row's output o.
     const int wq = warp & 3;
+    const int half = (warp - 6) >> 2;
     const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    constexpr int DH = D / 2;
     int po = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
@@ -838,31 +972,27 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
       int grow = bi.rt * BM + row;
       bool valid_row = grow < rows;
       int h = bi.kvh * L.g + (valid_row ? grow / tr.W : 0), w = valid_row ? grow % tr.W : 0;
-      float o[D];
+      float2 o2[DH / 2];
       float lsum = 0.0f, onorm = 0.0f;
       int nvis = 0;
-      if (valid_row) {
+      {
         const float *st = tr.stats + (((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4);
-        float4 hd = *reinterpret_cast<const float4 *>(st);
+        float4 hd = valid_row ? *reinterpret_cast<const float4 *>(st) : make_float4(0.f, 0.f, 0.f, 0.f);
         lsum = hd.y;
         nvis = (int)hd.z;
         float ss = 0.0f;
 #pragma unroll
         for (int c = 0; c < D; c += 4) {
-          float4 v = *reinterpret_cast<const float4 *>(st + 4 + c);
-          o[c] = v.x;
-          o[c + 1] = v.y;
-          o[c + 2] = v.z;
-          o[c + 3] = v.w;
+          float4 v = valid_row ? *reinterpret_cast<const float4 *>(st + 4 + c) : make_float4(0.f, 0.f, 0.f, 0.f);
           ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+          if ((c >> 6) == half) {
+            o2[(c & 63) / 2] = make_float2(v.x, v.y);
+            o2[(c & 63) / 2 + 1] = make_float2(v.z, v.w);
+          }
         }
         onorm = sqrtf(ss);
-      } else {
-#pragma unroll
-        for (int c = 0; c < D; ++c) o[c] = 0.0f;
       }
-      int npages = 0;
-      for (int E = bi.E0; E < bi.E1; ++E) npages += has_slots(tr, E);
+      int npages = tr.items[2 * bi.k + 1].x;
       for (int k = 0; k < npages && ok; ++k, ++po) {
         int a = po & 1, f = po % NFIFO;
         if (!mbar_wait(&sm.fifo_full[f], (po / NFIFO) & 1, kWait, abort_flag) ||
@@ -874,16 +1004,19 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
         float S_E = sm.fifo_s[f][row];
         int n_E = sm.fifo_n[f][row];
         int E = sm.fifo_page[f];
-        float num2 = 0.0f;
+        const float2 nS = make_float2(-S_E, -S_E);
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
+        for (int c0 = 0; c0 < DH; c0 += 32) {
           uint32_t r[32];
-          tmem_ld32(tm + lane_base + 2 * BT + a * D + c0, r);
+          tmem_ld32(tm + lane_base + 2 * BT + a * D + half * DH + c0, r);
           tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            float dlt = fmaf(-S_E, o[c0 + i], __uint_as_float(r[i]));
-            num2 = fmaf(dlt, dlt, num2);
+          for (int i = 0; i < 32; i += 4) {
+            float2 d0 = ffma2(nS, o2[(c0 + i) / 2], make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])));
+            float2 d1 = ffma2(nS, o2[(c0 + i) / 2 + 1], make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])));
+            acc0 = ffma2(d0, d0, acc0);
+            acc1 = ffma2(d1, d1, acc1);
           }
         }
         tc_fence_before();
@@ -892,12 +1025,31 @@ __global__ void __launch_bounds__(320, 1) pass_b_tc(const __grid_constant__ TcLa
           mbar_arrive(&sm.acc_empty[a]);
           mbar_arrive(&sm.fifo_empty[f]);
         }
-        float r = valid_row ? effect_value(n_E, nvis, S_E, lsum, num2, onorm) : 0.0f;
-        if (valid_row && tr.headR) atomic_max_nonneg(tr.headR + ((int64_t)bi.l * L.Hq + h) * tr.P + E, r);
-        float rm = r;
+        float part = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+        const int pb = po & 1;
+        if (half == 1) {  // hand the upper half to the lower warpgroup
+          if (po >= 2 && !mbar_wait(&sm.red_empty[pb], ((po >> 1) - 1) & 1, kWait, abort_flag)) {
+            ok = false;
+            break;
+          }
+          sm.red[pb][row] = part;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.red_full[pb]);
+        } else {
+          if (!mbar_wait(&sm.red_full[pb], (po >> 1) & 1, kWait, abort_flag)) {
+            ok = false;
+            break;
+          }
+          float num2 = part + sm.red[pb][row];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.red_empty[pb]);
+          float r = valid_row ? effect_value(n_E, nvis, S_E, lsum, num2, onorm) : 0.0f;
+          if (valid_row && tr.headR) atomic_max_nonneg(tr.headR + ((int64_t)bi.l * L.Hq + h) * tr.P + E, r);
+          float rm = r;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, off));
-        if (lane == 0) atomic_max_nonneg(tr.R + E, rm);
+          for (int off = 16; off > 0; off >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, off));
+          if (lane == 0) atomic_max_nonneg(tr.R + E, rm);
+        }
       }
     }
   }
@@ -953,10 +1105,12 @@ size_t smem_b() { return sizeof(SmemB) + 1024; }
 
 bool build_maps(TcMaps &mp, const TrajDev &t, int M, int H, int Hq) {
   uint64_t qrows = (uint64_t)M * Hq * (uint64_t)(t.W > 0 ? t.W : 1);
-  return map_q(&mp.q, t.q, qrows) && map_kv(&mp.k, t.k, t.S, H, M, t.st, t.sh, t.sl, BT) &&
-         map_kv(&mp.v, t.v, t.S, H, M, t.st, t.sh, t.sl, BT) &&
-         map_kv(&mp.kb, t.k, t.S, H, M, t.st, t.sh, t.sl, SLOT) &&
-         map_kv(&mp.vb, t.v, t.S, H, M, t.st, t.sh, t.sl, SLOT);
+  bool ok = map_q(&mp.q, t.q, qrows) && map_kv(&mp.k, t.k, t.S, H, M, t.st, t.sh, t.sl, BT) &&
+            map_kv(&mp.v, t.v, t.S, H, M, t.st, t.sh, t.sl, BT);
+  for (int i = 0; i < 3 && ok; ++i)
+    ok = map_kv(&mp.kb[i], t.k, t.S, H, M, t.st, t.sh, t.sl, SLOT << i) &&
+         map_kv(&mp.vb[i], t.v, t.S, H, M, t.st, t.sh, t.sl, SLOT << i);
+  return ok;
 }
 
 cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, int sm_count) {
@@ -964,13 +1118,13 @@ cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, in
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(pass_b_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_b());
   if (e != cudaSuccess) return e;
+  prep_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
   int na = L.item_off_a[L.n_traj];
   if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 192, smem_a(), s>>>(L, hdr);
   int rows = L.row_off[L.n_traj];
   if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
-  slots_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
   int nb = L.item_off_b[L.n_traj];
-  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 320, smem_b(), s>>>(L, hdr);
+  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 448, smem_b(), s>>>(L, hdr);
   return cudaGetLastError();
 }
 

@@ -13,14 +13,22 @@ constexpr int kRowsPerTile = 128;   // probe rows per MMA tile
 constexpr int kSlotsPerItem = 128;  // 16-token slots per pass-B work item
 
 struct TcMaps {
-  CUtensorMap q;       // Q as [M*Hq*W rows][128], box 64 x 128
-  CUtensorMap k, v;    // K, V as [M][H][S][128], box 64 x 128 x 1 x 1
-  CUtensorMap kb, vb;  // the same with 16-row boxes (page slots)
+  CUtensorMap q;             // Q as [M*Hq*W rows][128], box 64 x 128
+  CUtensorMap k, v;          // K, V as [M][H][S][128], box 64 x 128 x 1 x 1
+  CUtensorMap kb[3], vb[3];  // the same with 16-, 32- and 64-row boxes (runs of page slots)
+};
+
+// Per-trajectory facts computed once per call by the prep kernel.
+struct TcPrep {
+  int vis_all;  // leading resident tokens visible to every probe row
+  int pad[3];
 };
 
 struct TcTraj {
   const int32_t *pos, *qpos, *ps, *pl;
   int32_t *slot_off;  // workspace [P + 1]
+  int4 *items;        // workspace [nbitem][2]: {E0, E1, slot0, nslot}, {npages, 0, 0, 0}
+  TcPrep *prep;       // workspace
   float *stats;       // [M][Hq][W][132]
   float *R;           // [P]
   float *headR;       // [M][Hq][P] or null

@@ -94,3 +94,15 @@ def test_classify_and_compact_validation(lib):
     npend = (ctypes.c_int32 * 1)(100000)
     assert lib.commitkv_compact(ctypes.byref(shape), 1, trajs, ptrs, ptrs, npend, ptrs, ptrs, 10, 5, 4,
                                 ptrs, 0x3000, None, None, None, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
+
+
+def test_workspace_covers_smaller_caches(lib):
+    """A workspace sized for the post-commit caches serves the pre-commit
+    call too (its S and P are smaller), for every chunking regime."""
+    for dtype, d in ((ck.COMMITKV_BF16, 128), (ck.COMMITKV_F32, 64), (ck.COMMITKV_BF16, 64)):
+        shape = ck.Shape(4, 8, 32, d, dtype, 0.0)
+        for S_post in (300, 1500, 16384 + 2080, 36896, 139328):
+            big = lib.commitkv_workspace_size(ctypes.byref(shape), 1, (ck.Traj * 1)(_good_traj(S=S_post, W=32, P=S_post // 40, d=d, H=8)))
+            for S in range(max(1, S_post - 5000), S_post + 1, 97):
+                small = lib.commitkv_workspace_size(ctypes.byref(shape), 1, (ck.Traj * 1)(_good_traj(S=S, W=32, P=S // 40, d=d, H=8)))
+                assert 0 < small <= big, (d, S_post, S, small, big)

@@ -369,3 +369,30 @@ def test_scoring_paths_agree(name, seed, monkeypatch):
     a, s_ = out["tc"][1].reshape(-1, r.cfg.d + 4), out["simt"][1].reshape(-1, r.cfg.d + 4)
     assert np.array_equal(a[:, 2], s_[:, 2])
     _assert_close(a[:, 0], s_[:, 0], 1e-5, "row max")
+
+
+def test_many_zero_length_pages():
+    """Zero-length pages take no slot: an item may hold more pages than its
+    slots.  Their effect is 0; the other pages are unaffected."""
+    cfg = synth.small_config("zeros", L_pre=500, L_obs=40)
+    tr = synth.make_trajectory(cfg, 7)
+    ps, pl = [], []
+    for s_, l_ in zip(tr.page_start.tolist(), tr.page_len.tolist()):
+        for _ in range(12):  # zero-length pages at the page's start
+            ps.append(s_)
+            pl.append(0)
+        ps.append(s_)
+        pl.append(l_)
+    tr.page_start = np.asarray(ps, np.int32)
+    tr.page_len = np.asarray(pl, np.int32)
+    tr.eligible = np.ones(len(ps), np.uint8)
+    dev = DeviceTrajectory.upload(tr)
+    buf = StepBuffers(cfg, [dev])
+    buf.score_post()
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+    post = core.Problem(synth.values_f64(tr.K, "bf16"), synth.values_f64(tr.V, "bf16"), tr.pos,
+                        synth.values_f64(tr.Q_post, "bf16"), tr.qpos_post, tr.page_start, tr.page_len)
+    Rw, _ = core.page_effects(post, "explicit")
+    _assert_close(_np(buf.R_post[0]), Rw, 2e-2, "R+ with zero-length pages")
+    assert (_np(buf.R_post[0])[np.asarray(pl) == 0] == 0).all()
