@@ -14,7 +14,8 @@
  *
  * Conventions shared by every entry point
  *   - Memory: the caller owns all memory.  The library allocates nothing and
- *     keeps no global state.  Unless stated otherwise a pointer argument
+ *     keeps no global state (commitkv_compact_noalloc, at the end, is the
+ *     one exception: it keeps a fixed scratch array).  Unless stated otherwise a pointer argument
  *     is device memory; arrays of per-trajectory pointers ("host array of
  *     device pointers") and every struct argument are host memory and are
  *     read before the call returns.
@@ -54,6 +55,8 @@ typedef struct CUstream_st *cudaStream_t;
 
 #define COMMITKV_ABI_VERSION 1
 #define COMMITKV_MAX_TRAJ 64
+/* Size of the fixed device scratch of commitkv_compact_noalloc (4 MiB). */
+#define COMMITKV_NOALLOC_SCRATCH_BYTES (4u << 20)
 
 typedef enum {
   COMMITKV_OK = 0,
@@ -266,6 +269,51 @@ commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
                                  int32_t *const *idx_out, int32_t *n_idx_out,
                                  void *const *k_out, void *const *v_out, int32_t *const *pos_out,
                                  void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
+ * commitkv_compact without a workspace.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory where
+ * they compact.  A serving engine usually reserves nearly all device memory
+ * for its own KV pool at start-up, so a later cudaMalloc fails or has to go
+ * through an allocator that a plug-in cannot reach, and cudaFree
+ * synchronises the whole device.  This call allocates nothing: no
+ * cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * Same selection, outputs and host-side checks as commitkv_compact (all
+ * arguments but the workspace mean the same); its scratch is a fixed array
+ * of COMMITKV_NOALLOC_SCRATCH_BYTES (4 MiB) that the library keeps on every
+ * GPU that loads it, until the process exits.  Unlike the rest of this
+ * header, this is state held by the library:
+ *   - Limit: 256 + sum over trajectories of S_t rounded up to 256 must not
+ *     exceed COMMITKV_NOALLOC_SCRATCH_BYTES (one trajectory of up to
+ *     4,194,048 resident tokens); larger requests return
+ *     COMMITKV_ERR_WORKSPACE with nothing launched.
+ *   - Set-up: the first call with a given device current looks up the
+ *     array's device address (cudaGetSymbolAddress, which may also load the
+ *     library's device code on that device).  Make that first call before
+ *     any stream capture on that device.  A failed look-up returns
+ *     COMMITKV_ERR_CUDA.
+ *   - Sharing: every call on a device uses the same array.  Calls whose
+ *     work can overlap on the GPU (different streams, different host
+ *     threads) race on it and give wrong results; serialise them, for
+ *     example by issuing them all on one stream.
+ *   - Device-side errors: each call clears the array's status word first,
+ *     then the kernels record device-side input errors in it (as in the
+ *     workspace of commitkv_compact).  status_out, if not NULL, is a device
+ *     int32 that receives that word (a commitkv_status) once the call's work
+ *     is done on `stream`.
+ * -------------------------------------------------------------------- */
+commitkv_status commitkv_compact_noalloc(const commitkv_shape *shape, int32_t n_traj,
+                                         const commitkv_traj *cache,
+                                         const uint8_t *const *retired,
+                                         const int32_t *const *pending, const int32_t *n_pending,
+                                         const float *const *pending_priority,
+                                         const float *const *fill_score, int32_t budget_B,
+                                         int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                         int32_t *const *idx_out, int32_t *n_idx_out,
+                                         void *const *k_out, void *const *v_out,
+                                         int32_t *const *pos_out, int32_t *status_out,
+                                         cudaStream_t stream);
 
 #ifdef __cplusplus
 }
