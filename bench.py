@@ -287,9 +287,15 @@ def run_ours(args, rank, world, local):
 
 def buf_launches(buf):
     """Kernels of this library launched per step (counted from the launch
-    sequence of each call): scoring = pass A + combine + pass B per cache,
-    classify 1, joint test 1, compaction = select + gather."""
-    return 3 + 3 + 1 + 1 + 2
+    sequence of each call).  Scoring per cache: on the tensor-core path (bf16,
+    head_dim 128) prep + pass A + combine + pass B for every group of up to
+    16 trajectories, else pass A + combine + pass B; classify 1; joint test 1;
+    compaction = select + gather."""
+    cfg = buf.cfg
+    tc = cfg.dtype == "bf16" and cfg.d == 128 and os.environ.get("COMMITKV_SCORING") != "simt"
+    n = len(buf.trajs)
+    score = 4 * ((n + 15) // 16) if tc else 3
+    return 2 * score + 1 + 1 + 2
 
 
 def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):
