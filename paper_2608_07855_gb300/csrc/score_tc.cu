@@ -555,6 +555,8 @@ struct SmemB {
   int pg_len[kSlotsPerItem];
   int pg_slots[kSlotsPerItem];
   float red[2][BM];         // per page parity: the upper channel half of ||U - S o||^2
+  float ssum[SLOTS][BM];    // per softmax thread: slot sums of the current tile
+  int scnt[SLOTS][BM];      // and visible counts
   float fifo_s[NFIFO][BM];  // per page: S_E of every row
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
@@ -592,7 +594,7 @@ __device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
 
 __device__ __forceinline__ bool has_slots(const TcTraj &tr, int E) { return tr.slot_off[E + 1] > tr.slot_off[E]; }
 
-__global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+__global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   extern __shared__ uint8_t smem_raw[];
   SmemB &sm = *reinterpret_cast<SmemB *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -633,189 +635,197 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
   tc_fence_after();
   const uint32_t tm = sm.tmem;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    // The whole warp copies each item's page table into shared memory; lane 0
-    // then walks the slots and issues the copies.
-    uint64_t pol = policy_evict_first();
-    uint32_t it = 0, n_local = 0;
-    int po = 0;  // page ordinal
-    bool stop = false;
-    for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
-      if (*abort_flag) break;
-      ItemB bi = decode_b(L, item);
-      if (bi.nslot == 0) continue;
-      const TcTraj &tr = L.t[bi.t];
-      const TcMaps &mp = L.maps[bi.t];
-      // pages of the item; zero-length pages take no slot, so there may be more
-      // pages than the copy holds: those are read from global memory
-      int np = bi.E1 - bi.E0;
-      for (int e = lane; e < min(np, kSlotsPerItem); e += 32) {
-        int E = bi.E0 + e;
-        sm.pg_start[e] = tr.ps[E];
-        sm.pg_len[e] = tr.pl[E];
-        sm.pg_slots[e] = tr.slot_off[E + 1] - tr.slot_off[E];
-      }
-      __syncwarp();
-      if (lane == 0) {
-        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) {
-          stop = true;
-        } else {
-          mbar_expect_tx(&sm.q_full, kTileBytes);
-          int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
-          tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
-          tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
-          ++n_local;
-          // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
-          auto pslots = [&](int e) {
-            return e < kSlotsPerItem ? sm.pg_slots[e] : tr.slot_off[bi.E0 + e + 1] - tr.slot_off[bi.E0 + e];
-          };
-          int e = 0, sub = 0;
-          while (e < np && pslots(e) == 0) ++e;
-          int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-          for (int j = 0; j < ntile; ++j, ++it) {
-            int s = it % NST;
-            if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
-              stop = true;
-              break;
-            }
-            uint32_t bytes = 0;
-#pragma unroll
-            for (int q = 0; q < SLOTS; ++q) {
-              SlotMeta mt;
-              if (e < np) {
-                int pl = e < kSlotsPerItem ? sm.pg_len[e] : tr.pl[bi.E0 + e];
-                mt.tok0 = (e < kSlotsPerItem ? sm.pg_start[e] : tr.ps[bi.E0 + e]) + sub * SLOT;
-                mt.nv = min(SLOT, pl - sub * SLOT);
-                mt.po = po;
-                mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
-                sm.page_of[s][q] = bi.E0 + e;
-                bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
-                if (++sub * SLOT >= pl) {
-                  sub = 0;
-                  ++po;
-                  ++e;
-                  while (e < np && pslots(e) == 0) ++e;
-                }
-              } else {
-                mt.tok0 = 0;
-                mt.nv = 0;
-                mt.po = -1;
-                mt.flags = 0;
-                sm.page_of[s][q] = -1;
-              }
-              sm.meta[s][q] = mt;
-            }
-            // the slot table is written before the arrivals that publish it
-            mbar_expect_tx(&sm.k_full[s], bytes);
-            mbar_expect_tx(&sm.v_full[s], bytes);
-            // runs of slots whose rows are contiguous in memory (full pages
-            // of one event) travel as one box of 16, 32, 64 or 128 rows
-            int q = 0;
-            while (q < SLOTS) {
-              const SlotMeta m0 = sm.meta[s][q];
-              if (m0.po < 0) {
-                ++q;
-                continue;
-              }
-              int run = 1;
-              while (q + run < SLOTS && sm.meta[s][q + run].po >= 0 &&
-                     sm.meta[s][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s][q + run - 1].nv == SLOT)
-                ++run;
-              int done = 0;
-              while (done < run) {
-                int rem = run - done;
-                int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
-                if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
-                int tok = m0.tok0 + done * SLOT;
-                uint8_t *kd = sm.k[s] + (q + done) * SLOT * 128;
-                uint8_t *vd = sm.v[s] + (q + done) * SLOT * 128;
-                const CUtensorMap *km = lg == 3 ? &mp.k : &mp.kb[lg];
-                const CUtensorMap *vm = lg == 3 ? &mp.v : &mp.vb[lg];
-                tma4(kd, km, 0, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
-                tma4(kd + kHalf, km, 64, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
-                tma4(vd, vm, 0, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
-                tma4(vd + kHalf, vm, 64, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
-                done += 1 << lg;
-              }
-              q += run;
-            }
-          }
-        }
-      }
-      stop = __shfl_sync(0xffffffffu, stop, 0);
-      __syncwarp();
-    }
-    if (lane == 0 && *abort_flag) {
-      for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
-        mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
-        mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
-      }
-      if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+  // warpgroup 0: TMA producer, MMA issuer and two idle warps; 1: softmax;
+  // 2 and 3: epilogue.  Each branch first sets its warpgroup's register
+  // budget: 56 + 136 + 2 x 160 per thread = the launch's 4 x 128.
+  if (warp < 4) {
+    regs_dec<56>();  // warps 2 and 3 stay idle
+    if (warp == 0) {
+      // ------------------------------------------------------------ TMA producer
+      // The whole warp copies each item's page table into shared memory; lane 0
+      // then walks the slots and issues the copies.
+      uint64_t pol = policy_evict_first();
       uint32_t it = 0, n_local = 0;
-      bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      int po = 0;  // page ordinal
+      bool stop = false;
+      for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
+        if (*abort_flag) break;
         ItemB bi = decode_b(L, item);
         if (bi.nslot == 0) continue;
-        int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-        if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
-        ++n_local;
-        tc_fence_after();
-        auto qk = [&](uint32_t g) -> bool {
-          int s = g % NST, b = g & 1;
-          if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
-          if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
-          tc_fence_after();
-          issue_qk(tm, sm.q, sm.k[s], b);
-          mma_commit(&sm.s_full[b]);
-          return true;
-        };
-        ok = qk(it);
-        for (int j = 0; j < ntile && ok; ++j) {
-          uint32_t g = it + j;
-          if (j + 1 < ntile) {
-            ok = qk(g + 1);
-            if (!ok) break;
+        const TcTraj &tr = L.t[bi.t];
+        const TcMaps &mp = L.maps[bi.t];
+        // pages of the item; zero-length pages take no slot, so there may be more
+        // pages than the copy holds: those are read from global memory
+        int np = bi.E1 - bi.E0;
+        for (int e = lane; e < min(np, kSlotsPerItem); e += 32) {
+          int E = bi.E0 + e;
+          sm.pg_start[e] = tr.ps[E];
+          sm.pg_len[e] = tr.pl[E];
+          sm.pg_slots[e] = tr.slot_off[E + 1] - tr.slot_off[E];
+        }
+        __syncwarp();
+        if (lane == 0) {
+          if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) {
+            stop = true;
           } else {
-            mma_commit(&sm.q_empty);
-          }
-          int s = g % NST, b = g & 1;
-          if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
-              !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          for (int q = 0; q < SLOTS && ok; ++q) {
-            SlotMeta mt = sm.meta[s][q];
-            if (mt.po < 0) continue;
-            int a = mt.po & 1;
-            if ((mt.flags & 1) && mt.po >= 2) {
-              if (!mbar_wait(&sm.acc_empty[a], ((mt.po >> 1) - 1) & 1, kWait, abort_flag)) {
-                ok = false;
+            mbar_expect_tx(&sm.q_full, kTileBytes);
+            int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
+            tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+            tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
+            ++n_local;
+            // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
+            auto pslots = [&](int e) {
+              return e < kSlotsPerItem ? sm.pg_slots[e] : tr.slot_off[bi.E0 + e + 1] - tr.slot_off[bi.E0 + e];
+            };
+            int e = 0, sub = 0;
+            while (e < np && pslots(e) == 0) ++e;
+            int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+            for (int j = 0; j < ntile; ++j, ++it) {
+              int s = it % NST;
+              if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
+                stop = true;
                 break;
               }
-              tc_fence_after();
+              uint32_t bytes = 0;
+#pragma unroll 1
+              for (int q = 0; q < SLOTS; ++q) {
+                SlotMeta mt;
+                if (e < np) {
+                  int pl = e < kSlotsPerItem ? sm.pg_len[e] : tr.pl[bi.E0 + e];
+                  mt.tok0 = (e < kSlotsPerItem ? sm.pg_start[e] : tr.ps[bi.E0 + e]) + sub * SLOT;
+                  mt.nv = min(SLOT, pl - sub * SLOT);
+                  mt.po = po;
+                  mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
+                  sm.page_of[s][q] = bi.E0 + e;
+                  bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
+                  if (++sub * SLOT >= pl) {
+                    sub = 0;
+                    ++po;
+                    ++e;
+                    while (e < np && pslots(e) == 0) ++e;
+                  }
+                } else {
+                  mt.tok0 = 0;
+                  mt.nv = 0;
+                  mt.po = -1;
+                  mt.flags = 0;
+                  sm.page_of[s][q] = -1;
+                }
+                sm.meta[s][q] = mt;
+              }
+              // the slot table is written before the arrivals that publish it
+              mbar_expect_tx(&sm.k_full[s], bytes);
+              mbar_expect_tx(&sm.v_full[s], bytes);
+              // runs of slots whose rows are contiguous in memory (full pages
+              // of one event) travel as one box of 16, 32, 64 or 128 rows
+              int q = 0;
+              while (q < SLOTS) {
+                const SlotMeta m0 = sm.meta[s][q];
+                if (m0.po < 0) {
+                  ++q;
+                  continue;
+                }
+                int run = 1;
+                while (q + run < SLOTS && sm.meta[s][q + run].po >= 0 &&
+                       sm.meta[s][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s][q + run - 1].nv == SLOT)
+                  ++run;
+                int done = 0;
+                while (done < run) {
+                  int rem = run - done;
+                  int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
+                  if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
+                  int tok = m0.tok0 + done * SLOT;
+                  uint8_t *kd = sm.k[s] + (q + done) * SLOT * 128;
+                  uint8_t *vd = sm.v[s] + (q + done) * SLOT * 128;
+                  const CUtensorMap *km = lg == 3 ? &mp.k : &mp.kb[lg];
+                  const CUtensorMap *vm = lg == 3 ? &mp.v : &mp.vb[lg];
+                  tma4(kd, km, 0, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
+                  tma4(kd + kHalf, km, 64, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
+                  tma4(vd, vm, 0, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
+                  tma4(vd + kHalf, vm, 64, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
+                  done += 1 << lg;
+                }
+                q += run;
+              }
             }
-            issue_pv_step(tm, 2 * BT + a * D, sm.v[s], b, q, (mt.flags & 1) != 0);
-            if (mt.flags & 2) mma_commit(&sm.acc_full[a]);
           }
-          mma_commit(&sm.s_empty[b]);
-          mma_commit(&sm.kv_empty[s]);
         }
-        it += ntile;
+        stop = __shfl_sync(0xffffffffu, stop, 0);
+        __syncwarp();
       }
-      if (*abort_flag) {
-        mma_commit(&sm.drain);
-        mbar_wait_drain(&sm.drain, 0, kWait);
+      if (lane == 0 && *abort_flag) {
+        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
+          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
+          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
+        }
+        if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
+      }
+    } else if (warp == 1) {
+      // ------------------------------------------------------------ MMA issuer
+      if (lane == 0) {
+        uint32_t it = 0, n_local = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+          ItemB bi = decode_b(L, item);
+          if (bi.nslot == 0) continue;
+          int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+          if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
+          ++n_local;
+          tc_fence_after();
+          auto qk = [&](uint32_t g) -> bool {
+            int s = g % NST, b = g & 1;
+            if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
+            if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
+            tc_fence_after();
+            issue_qk(tm, sm.q, sm.k[s], b);
+            mma_commit(&sm.s_full[b]);
+            return true;
+          };
+          ok = qk(it);
+          for (int j = 0; j < ntile && ok; ++j) {
+            uint32_t g = it + j;
+            if (j + 1 < ntile) {
+              ok = qk(g + 1);
+              if (!ok) break;
+            } else {
+              mma_commit(&sm.q_empty);
+            }
+            int s = g % NST, b = g & 1;
+            if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
+                !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll 1
+            for (int q = 0; q < SLOTS && ok; ++q) {
+              SlotMeta mt = sm.meta[s][q];
+              if (mt.po < 0) continue;
+              int a = mt.po & 1;
+              if ((mt.flags & 1) && mt.po >= 2) {
+                if (!mbar_wait(&sm.acc_empty[a], ((mt.po >> 1) - 1) & 1, kWait, abort_flag)) {
+                  ok = false;
+                  break;
+                }
+                tc_fence_after();
+              }
+              issue_pv_step(tm, 2 * BT + a * D, sm.v[s], b, q, (mt.flags & 1) != 0);
+              if (mt.flags & 2) mma_commit(&sm.acc_full[a]);
+            }
+            mma_commit(&sm.s_empty[b]);
+            mma_commit(&sm.kv_empty[s]);
+          }
+          it += ntile;
+        }
+        if (*abort_flag) {
+          mma_commit(&sm.drain);
+          mbar_wait_drain(&sm.drain, 0, kWait);
+        }
       }
     }
-  } else if (warp < 6) {
-    // ------------------------------------------------------------ softmax (warps 2..5)
+  } else if (warp < 8) {
+    // ------------------------------------------------------------ softmax (warps 4..7)
+    regs_inc<136>();
     const int wq = warp & 3;
     const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
@@ -852,14 +862,14 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
         }
         // slots inside the prefix every probe row sees need no position test
         bool full = true;
-#pragma unroll
+#pragma unroll 1
         for (int q = 0; q < SLOTS; ++q) {
           const SlotMeta mt = sm.meta[s][q];
           full &= mt.po < 0 || mt.tok0 + mt.nv <= vis_all;
         }
         if (!full) {  // each warp keeps its own copy: no cross-warp barrier
           __syncwarp();
-#pragma unroll
+#pragma unroll 1
           for (int c = lane; c < BT; c += 32) {
             const SlotMeta mt = sm.meta[s][c / SLOT];
             int i = c % SLOT;
@@ -872,60 +882,52 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
           break;
         }
         tc_fence_after();
-        // e = exp(s - m) on the visible page tokens; fp32 slot sums; P as the
-        // (hi, lo) bf16 pair written over the S columns just read
-        float slot_s[SLOTS];
-        int slot_n[SLOTS];
-        // 32-column chunks, software-pipelined: the load of chunk c + 1 is in
-        // flight while chunk c is computed (scores in, probabilities out, in place)
-        float eb[2][32];
-        tmem_ld32f(tm + lane_base + b * BT, eb[0]);
-        tmem_wait_ld();
-#pragma unroll
+        // Per 32-column chunk (two slots): e = exp(s - m) on the visible page
+        // tokens (a visibility bit mask turns the others into -inf, so e = 0);
+        // per-slot sums and counts to shared memory; P as the (hi, lo) bf16
+        // pair written over the S columns just read.  The chunk loop is not
+        // unrolled: a small loop body keeps the instruction cache warm.
+#pragma unroll 1
         for (int ch = 0; ch < BT / 32; ++ch) {
-          float *e = eb[ch & 1];
-          if (ch + 1 < BT / 32) tmem_ld32f(tm + lane_base + b * BT + 32 * (ch + 1), eb[(ch + 1) & 1]);
-#pragma unroll
-          for (int h2 = 0; h2 < 2; ++h2) {
-            const int q = 2 * ch + h2;
-            const int nv = sm.meta[s][q].nv;
-            float *es = e + h2 * SLOT;
-            int nn;
-            if (full && nv == SLOT) {
-#pragma unroll
-              for (int i = 0; i < SLOT; ++i) es[i] = fast_exp2(fmaf(es[i], L.scale_log2, neg_m2));
-              nn = valid_row ? SLOT : 0;
-            } else {
-              nn = 0;
-#pragma unroll
-              for (int i = 0; i < SLOT; ++i) {
-                bool vis = i < nv && (full || sm.pos[wq][32 * ch + h2 * SLOT + i] <= qp);
-                es[i] = vis ? fast_exp2(fmaf(es[i], L.scale_log2, neg_m2)) : 0.0f;
-                nn += vis && valid_row;
-              }
-            }
-            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll
-            for (int i = 0; i < SLOT; i += 4) {
-              a0 += es[i];
-              a1 += es[i + 1];
-              a2 += es[i + 2];
-              a3 += es[i + 3];
-            }
-            slot_s[q] = (a0 + a1) + (a2 + a3);
-            slot_n[q] = nn;
+          float x[32];
+          tmem_ld32f(tm + lane_base + b * BT + 32 * ch, x);
+          const int nv0 = sm.meta[s][2 * ch].nv, nv1 = sm.meta[s][2 * ch + 1].nv;
+          uint32_t vm = (nv0 >= SLOT ? 0xffffu : (1u << max(nv0, 0)) - 1u) |
+                        ((nv1 >= SLOT ? 0xffffu : (1u << max(nv1, 0)) - 1u) << 16);
+          if (!full) {
+#pragma unroll 1
+            for (int i = 0; i < 32; ++i)
+              if (sm.pos[wq][32 * ch + i] > qp) vm &= ~(1u << i);
           }
+          if (!valid_row) vm = 0;
+          tmem_wait_ld();
+          float a0 = 0.f, a1 = 0.f, c0 = 0.f, c1 = 0.f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float xi = (vm >> i) & 1u ? x[i] : -INFINITY;
+            x[i] = fast_exp2(fmaf(xi, L.scale_log2, neg_m2));
+          }
+#pragma unroll
+          for (int i = 0; i < 16; i += 2) {
+            a0 += x[i];
+            a1 += x[i + 1];
+            c0 += x[16 + i];
+            c1 += x[17 + i];
+          }
+          sm.ssum[2 * ch][row] = a0 + a1;
+          sm.ssum[2 * ch + 1][row] = c0 + c1;
+          sm.scnt[2 * ch][row] = __popc(vm & 0xffffu);
+          sm.scnt[2 * ch + 1][row] = __popc(vm >> 16);
           uint32_t pk[32];
-          split_pack32(e, pk);
+          split_pack32(x, pk);
           tmem_st32(tm + lane_base + b * BT + 32 * ch, pk);
-          if (ch + 1 < BT / 32) tmem_wait_ld();
         }
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.p_full);
         // page sums: walk the slots in order, hand finished pages to the epilogue
-#pragma unroll
+#pragma unroll 1
         for (int q = 0; q < SLOTS; ++q) {
           const SlotMeta mt = sm.meta[s][q];
           if (mt.po < 0 || !ok) continue;
@@ -933,8 +935,8 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
             S_cur = 0.0f;
             n_cur = 0;
           }
-          S_cur += slot_s[q];
-          n_cur += slot_n[q];
+          S_cur += sm.ssum[q][row];
+          n_cur += sm.scnt[q][row];
           if (mt.flags & 2) {
             int f = po_seen % NFIFO;
             if (po_seen >= NFIFO &&
@@ -954,11 +956,12 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
       it += ntile;
     }
   } else {
-    // ------------------------------------------------------------ epilogue (warps 6..13)
+    // ------------------------------------------------------------ epilogue (warps 8..15)
     // Two warpgroups split the 128 channels; each thread owns one row and 64
     // channels of that row's output o.
+    regs_inc<160>();
     const int wq = warp & 3;
-    const int half = (warp - 6) >> 2;
+    const int half = (warp - 8) >> 2;
     const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
     constexpr int DH = D / 2;
@@ -1005,25 +1008,29 @@ __global__ void __launch_bounds__(448, 1) pass_b_tc(const __grid_constant__ TcLa
         int n_E = sm.fifo_n[f][row];
         int E = sm.fifo_page[f];
         const float2 nS = make_float2(-S_E, -S_E);
-        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
-#pragma unroll
-        for (int c0 = 0; c0 < DH; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32(tm + lane_base + 2 * BT + a * D + half * DH + c0, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; i += 4) {
-            float2 d0 = ffma2(nS, o2[(c0 + i) / 2], make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])));
-            float2 d1 = ffma2(nS, o2[(c0 + i) / 2 + 1], make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])));
-            acc0 = ffma2(d0, d0, acc0);
-            acc1 = ffma2(d1, d1, acc1);
-          }
-        }
+        // copy this half of U_E out of TMEM, then hand the accumulator back
+        uint32_t r0[32], r1[32];
+        tmem_ld64(tm + lane_base + 2 * BT + a * D + half * DH, r0, r1);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&sm.acc_empty[a]);
           mbar_arrive(&sm.fifo_empty[f]);
+        }
+        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < 32; i += 4) {
+          float2 d0 = ffma2(nS, o2[i / 2], make_float2(__uint_as_float(r0[i]), __uint_as_float(r0[i + 1])));
+          float2 d1 = ffma2(nS, o2[i / 2 + 1], make_float2(__uint_as_float(r0[i + 2]), __uint_as_float(r0[i + 3])));
+          acc0 = ffma2(d0, d0, acc0);
+          acc1 = ffma2(d1, d1, acc1);
+        }
+#pragma unroll
+        for (int i = 0; i < 32; i += 4) {
+          float2 d0 = ffma2(nS, o2[16 + i / 2], make_float2(__uint_as_float(r1[i]), __uint_as_float(r1[i + 1])));
+          float2 d1 = ffma2(nS, o2[16 + i / 2 + 1], make_float2(__uint_as_float(r1[i + 2]), __uint_as_float(r1[i + 3])));
+          acc0 = ffma2(d0, d0, acc0);
+          acc1 = ffma2(d1, d1, acc1);
         }
         float part = (acc0.x + acc0.y) + (acc1.x + acc1.y);
         const int pb = po & 1;
@@ -1124,7 +1131,7 @@ cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, in
   int rows = L.row_off[L.n_traj];
   if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
   int nb = L.item_off_b[L.n_traj];
-  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 448, smem_b(), s>>>(L, hdr);
+  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 512, smem_b(), s>>>(L, hdr);
   return cudaGetLastError();
 }
 

@@ -281,6 +281,19 @@ __device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&a)[32], uin
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Per-warpgroup register budget (PTX setmaxnreg; every warp of the
+// warpgroup executes the same instruction).  The increases of a block must
+// not exceed what its decreases release: threads x registers at launch is
+// the whole pool.
+template <int N>
+__device__ __forceinline__ void regs_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void regs_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
