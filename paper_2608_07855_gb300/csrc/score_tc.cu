@@ -35,7 +35,9 @@ using namespace ckv::sm103;
 constexpr int D = 128;
 constexpr int BM = 128;  // probe rows per tile (MMA M)
 constexpr int BT = 128;  // KV rows per tile (MMA N of Q K^T, K of P V)
-constexpr int NST = 2;   // K/V pipeline stages
+constexpr int NST = 2;   // K/V pipeline stages (pass A)
+constexpr int NKB = 3;   // pass B: K stages (with their slot tables)
+constexpr int NVB = 2;   // pass B: V stages
 constexpr int SLOT = 16;
 constexpr int SLOTS = BT / SLOT;  // slots per pass-B tile
 constexpr int NFIFO = 8;          // page-sum FIFO depth (>= SLOTS)
@@ -546,10 +548,11 @@ struct SlotMeta {
 
 struct SmemB {
   alignas(1024) uint8_t q[kTileBytes];
-  alignas(1024) uint8_t k[NST][kTileBytes];
-  alignas(1024) uint8_t v[NST][kTileBytes];
-  SlotMeta meta[NST][SLOTS];
-  int page_of[NST][SLOTS];  // page id of each slot
+  alignas(1024) uint8_t k[NKB][kTileBytes];
+  alignas(1024) uint8_t v[NVB][kTileBytes];
+  SlotMeta meta[NKB][SLOTS];
+  int page_of[NKB][SLOTS];  // page id of each slot
+  uint32_t tile_bytes[NKB]; // bytes of the tile's K (and V) copies
   int pos[4][BT];           // per softmax warp: positions of the current tile
   int pg_start[kSlotsPerItem];  // the producer's copy of the item's page table
   int pg_len[kSlotsPerItem];
@@ -560,8 +563,9 @@ struct SmemB {
   float fifo_s[NFIFO][BM];  // per page: S_E of every row
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
-  uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full,
-      acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], red_full[2], red_empty[2], drain;
+  uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], meta_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2],
+      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], red_full[2],
+      red_empty[2], drain;
   uint32_t tmem;
   int abort_flag;
 };
@@ -605,10 +609,14 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     sm.abort_flag = 0;
     mbar_init(&sm.q_full, 1);
     mbar_init(&sm.q_empty, 1);
-    for (int s = 0; s < NST; ++s) {
+    for (int s = 0; s < NKB; ++s) {
       mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
+      mbar_init(&sm.meta_empty[s], 5);  // four softmax warps and the MMA thread
+    }
+    for (int s = 0; s < NVB; ++s) {
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.v_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.s_full[b], 1);
@@ -645,7 +653,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       // The whole warp copies each item's page table into shared memory; lane 0
       // then walks the slots and issues the copies.
       uint64_t pol = policy_evict_first();
-      uint32_t it = 0, n_local = 0;
+      uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
       int po = 0;  // page ordinal
       bool stop = false;
       for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
@@ -679,13 +687,43 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             };
             int e = 0, sub = 0;
             while (e < np && pslots(e) == 0) ++e;
-            int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-            for (int j = 0; j < ntile; ++j, ++it) {
-              int s = it % NST;
-              if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
-                stop = true;
-                break;
+            // runs of slots whose rows are contiguous in memory (full pages of
+            // one event) travel as one box of 16, 32, 64 or 128 rows
+            auto issue_boxes = [&](int s3, uint8_t *dst, const CUtensorMap *big, const CUtensorMap *small,
+                                   uint64_t *bar) {
+              int q = 0;
+              while (q < SLOTS) {
+                const SlotMeta m0 = sm.meta[s3][q];
+                if (m0.po < 0) {
+                  ++q;
+                  continue;
+                }
+                int run = 1;
+                while (q + run < SLOTS && sm.meta[s3][q + run].po >= 0 &&
+                       sm.meta[s3][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s3][q + run - 1].nv == SLOT)
+                  ++run;
+                int done = 0;
+                while (done < run) {
+                  int rem = run - done;
+                  int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
+                  if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
+                  int tok = m0.tok0 + done * SLOT;
+                  uint8_t *d = dst + (q + done) * SLOT * 128;
+                  const CUtensorMap *m = lg == 3 ? big : small + lg;
+                  tma4(d, m, 0, tok, bi.kvh, bi.l, bar, pol);
+                  tma4(d + kHalf, m, 64, tok, bi.kvh, bi.l, bar, pol);
+                  done += 1 << lg;
+                }
+                q += run;
               }
+            };
+            // K of tile g (and its slot table) once Q K^T of tile g - 3 is done and
+            // its slot table released
+            auto load_k = [&](uint32_t g) -> bool {
+              int s3 = g % NKB;
+              if (g >= NKB && (!mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag) ||
+                               !mbar_wait(&sm.meta_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)))
+                return false;
               uint32_t bytes = 0;
 #pragma unroll 1
               for (int q = 0; q < SLOTS; ++q) {
@@ -696,7 +734,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                   mt.nv = min(SLOT, pl - sub * SLOT);
                   mt.po = po;
                   mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
-                  sm.page_of[s][q] = bi.E0 + e;
+                  sm.page_of[s3][q] = bi.E0 + e;
                   bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
                   if (++sub * SLOT >= pl) {
                     sub = 0;
@@ -709,55 +747,45 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                   mt.nv = 0;
                   mt.po = -1;
                   mt.flags = 0;
-                  sm.page_of[s][q] = -1;
+                  sm.page_of[s3][q] = -1;
                 }
-                sm.meta[s][q] = mt;
+                sm.meta[s3][q] = mt;
               }
-              // the slot table is written before the arrivals that publish it
-              mbar_expect_tx(&sm.k_full[s], bytes);
-              mbar_expect_tx(&sm.v_full[s], bytes);
-              // runs of slots whose rows are contiguous in memory (full pages
-              // of one event) travel as one box of 16, 32, 64 or 128 rows
-              int q = 0;
-              while (q < SLOTS) {
-                const SlotMeta m0 = sm.meta[s][q];
-                if (m0.po < 0) {
-                  ++q;
-                  continue;
-                }
-                int run = 1;
-                while (q + run < SLOTS && sm.meta[s][q + run].po >= 0 &&
-                       sm.meta[s][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s][q + run - 1].nv == SLOT)
-                  ++run;
-                int done = 0;
-                while (done < run) {
-                  int rem = run - done;
-                  int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
-                  if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
-                  int tok = m0.tok0 + done * SLOT;
-                  uint8_t *kd = sm.k[s] + (q + done) * SLOT * 128;
-                  uint8_t *vd = sm.v[s] + (q + done) * SLOT * 128;
-                  const CUtensorMap *km = lg == 3 ? &mp.k : &mp.kb[lg];
-                  const CUtensorMap *vm = lg == 3 ? &mp.v : &mp.vb[lg];
-                  tma4(kd, km, 0, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
-                  tma4(kd + kHalf, km, 64, tok, bi.kvh, bi.l, &sm.k_full[s], pol);
-                  tma4(vd, vm, 0, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
-                  tma4(vd + kHalf, vm, 64, tok, bi.kvh, bi.l, &sm.v_full[s], pol);
-                  done += 1 << lg;
-                }
-                q += run;
-              }
+              sm.tile_bytes[s3] = bytes;
+              // the slot table is written before the arrival that publishes it
+              mbar_expect_tx(&sm.k_full[s3], bytes);
+              issue_boxes(s3, sm.k[s3], &mp.k, mp.kb, &sm.k_full[s3]);
+              ++n_k;
+              return true;
+            };
+            // V of tile g once P V of tile g - 2 is done
+            auto load_v = [&](uint32_t g) -> bool {
+              int s3 = g % NKB, s2 = g % NVB;
+              if (g >= NVB && !mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag)) return false;
+              mbar_expect_tx(&sm.v_full[s2], sm.tile_bytes[s3]);
+              issue_boxes(s3, sm.v[s2], &mp.v, mp.vb, &sm.v_full[s2]);
+              ++n_v;
+              return true;
+            };
+            // K runs one tile ahead of V
+            int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+            stop = !load_k(it);
+            for (int j = 0; j < ntile && !stop; ++j) {
+              if (j + 1 < ntile && !load_k(it + j + 1)) stop = true;
+              else if (!load_v(it + j)) stop = true;
             }
+            it += ntile;
           }
         }
         stop = __shfl_sync(0xffffffffu, stop, 0);
         __syncwarp();
       }
       if (lane == 0 && *abort_flag) {
-        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
-          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
-          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
-        }
+        // let the copies already issued land before the CTA leaves
+        for (uint32_t u = (n_k > NKB ? n_k - NKB : 0); u < n_k; ++u)
+          mbar_wait_drain(&sm.k_full[u % NKB], (u / NKB) & 1, kWait);
+        for (uint32_t u = (n_v > NVB ? n_v - NVB : 0); u < n_v; ++u)
+          mbar_wait_drain(&sm.v_full[u % NVB], (u / NVB) & 1, kWait);
         if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
       }
     } else if (warp == 1) {
@@ -772,34 +800,41 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
           ++n_local;
           tc_fence_after();
-          auto qk = [&](uint32_t g) -> bool {
-            int s = g % NST, b = g & 1;
-            if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
+          auto qk = [&](uint32_t g, int j) -> bool {
+            int s3 = g % NKB, b = g & 1;
+            if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag)) return false;
             if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
             tc_fence_after();
-            issue_qk(tm, sm.q, sm.k[s], b);
+            issue_qk(tm, sm.q, sm.k[s3], b);
             mma_commit(&sm.s_full[b]);
+            mma_commit(&sm.k_empty[s3]);
+            if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
             return true;
           };
-          ok = qk(it);
+          ok = qk(it, 0);
           for (int j = 0; j < ntile && ok; ++j) {
             uint32_t g = it + j;
+            int s3 = g % NKB, s2 = g % NVB, b = g & 1;
+            // Q K^T of the next tile goes first when its operands are already there
+            bool next_issued = false;
             if (j + 1 < ntile) {
-              ok = qk(g + 1);
-              if (!ok) break;
-            } else {
-              mma_commit(&sm.q_empty);
+              uint32_t g1 = g + 1;
+              if (mbar_try_wait(&sm.k_full[g1 % NKB], (g1 / NKB) & 1) &&
+                  (g1 < 2 || mbar_try_wait(&sm.s_empty[g1 & 1], ((g1 >> 1) - 1) & 1))) {
+                ok = qk(g1, j + 1);
+                next_issued = true;
+                if (!ok) break;
+              }
             }
-            int s = g % NST, b = g & 1;
             if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
-                !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
+                !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
               ok = false;
               break;
             }
             tc_fence_after();
 #pragma unroll 1
             for (int q = 0; q < SLOTS && ok; ++q) {
-              SlotMeta mt = sm.meta[s][q];
+              SlotMeta mt = sm.meta[s3][q];
               if (mt.po < 0) continue;
               int a = mt.po & 1;
               if ((mt.flags & 1) && mt.po >= 2) {
@@ -809,11 +844,13 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                 }
                 tc_fence_after();
               }
-              issue_pv_step(tm, 2 * BT + a * D, sm.v[s], b, q, (mt.flags & 1) != 0);
+              issue_pv_step(tm, 2 * BT + a * D, sm.v[s2], b, q, (mt.flags & 1) != 0);
               if (mt.flags & 2) mma_commit(&sm.acc_full[a]);
             }
             mma_commit(&sm.s_empty[b]);
-            mma_commit(&sm.kv_empty[s]);
+            mma_commit(&sm.v_empty[s2]);
+            mbar_arrive(&sm.meta_empty[s3]);  // done with the slot table
+            if (ok && j + 1 < ntile && !next_issued) ok = qk(g + 1, j + 1);
           }
           it += ntile;
         }
@@ -854,9 +891,9 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
       for (int j = 0; j < ntile && ok; ++j) {
         uint32_t g = it + j;
-        int s = g % NST, b = g & 1;
+        int s = g % NKB, b = g & 1;
         // the slot table of this stage is published with its K copies
-        if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) {
+        if (!mbar_wait(&sm.k_full[s], (g / NKB) & 1, kWait, abort_flag)) {
           ok = false;
           break;
         }
@@ -952,6 +989,8 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             ++po_seen;
           }
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.meta_empty[s]);  // done with the slot table
       }
       it += ntile;
     }
