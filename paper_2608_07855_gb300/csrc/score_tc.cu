@@ -80,11 +80,11 @@ __device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int ks) {
 // of P_lo), O at 256.
 struct SmemA {
   alignas(1024) uint8_t q[kTileBytes];
-  alignas(1024) uint8_t k[NST][kTileBytes];
-  alignas(1024) uint8_t v[NST][kTileBytes];
+  alignas(1024) uint8_t k[NKB][kTileBytes];
+  alignas(1024) uint8_t v[NVB][kTileBytes];
   int pos[4][BT];  // per softmax warp: positions of the current tile
-  uint64_t q_full, q_empty, k_full[NST], v_full[NST], kv_empty[NST], s_full[2], s_empty[2], p_full, pv_done,
-      o_full, o_empty, drain;
+  uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2], s_empty[2], p_full,
+      pv_done, o_full, o_empty, drain;
   uint32_t tmem;
   int abort_flag;
 };
@@ -141,10 +141,13 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
     sm.abort_flag = 0;
     mbar_init(&sm.q_full, 1);
     mbar_init(&sm.q_empty, 1);
-    for (int s = 0; s < NST; ++s) {
+    for (int s = 0; s < NKB; ++s) {
       mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
+    }
+    for (int s = 0; s < NVB; ++s) {
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.v_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.s_full[b], 1);
@@ -170,8 +173,9 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       uint64_t pol = policy_evict_normal();
-      uint32_t it = 0, n_local = 0;
-      for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++n_local) {
+      uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
+      bool stop = false;
+      for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x, ++n_local) {
         if (*abort_flag) break;
         ItemA a = decode_a(L, item);
         const TcTraj &tr = L.t[a.t];
@@ -182,28 +186,40 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
         tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
         int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
-        bool stop = false;
-        for (int tok = t0; tok < t1; tok += BT, ++it) {
-          int s = it % NST;
-          if (it >= NST && !mbar_wait(&sm.kv_empty[s], ((it / NST) - 1) & 1, kWait, abort_flag)) {
-            stop = true;
-            break;
-          }
-          mbar_expect_tx(&sm.k_full[s], kTileBytes);
-          tma4(sm.k[s], &mp.k, 0, tok, a.kvh, a.l, &sm.k_full[s], pol);
-          tma4(sm.k[s] + kHalf, &mp.k, 64, tok, a.kvh, a.l, &sm.k_full[s], pol);
-          mbar_expect_tx(&sm.v_full[s], kTileBytes);
-          tma4(sm.v[s], &mp.v, 0, tok, a.kvh, a.l, &sm.v_full[s], pol);
-          tma4(sm.v[s] + kHalf, &mp.v, 64, tok, a.kvh, a.l, &sm.v_full[s], pol);
+        int ntile = (t1 - t0 + BT - 1) / BT;
+        // K of tile g once Q K^T of tile g - 3 is done; V once P V of tile g - 2 is
+        auto load_k = [&](uint32_t g, int tok) -> bool {
+          int s3 = g % NKB;
+          if (g >= NKB && !mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)) return false;
+          mbar_expect_tx(&sm.k_full[s3], kTileBytes);
+          tma4(sm.k[s3], &mp.k, 0, tok, a.kvh, a.l, &sm.k_full[s3], pol);
+          tma4(sm.k[s3] + kHalf, &mp.k, 64, tok, a.kvh, a.l, &sm.k_full[s3], pol);
+          ++n_k;
+          return true;
+        };
+        auto load_v = [&](uint32_t g, int tok) -> bool {
+          int s2 = g % NVB;
+          if (g >= NVB && !mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag)) return false;
+          mbar_expect_tx(&sm.v_full[s2], kTileBytes);
+          tma4(sm.v[s2], &mp.v, 0, tok, a.kvh, a.l, &sm.v_full[s2], pol);
+          tma4(sm.v[s2] + kHalf, &mp.v, 64, tok, a.kvh, a.l, &sm.v_full[s2], pol);
+          ++n_v;
+          return true;
+        };
+        // K runs one tile ahead of V
+        if (ntile > 0) stop = !load_k(it, t0);
+        for (int j = 0; j < ntile && !stop; ++j) {
+          if (j + 1 < ntile && !load_k(it + j + 1, t0 + (j + 1) * BT)) stop = true;
+          else if (!load_v(it + j, t0 + j * BT)) stop = true;
         }
-        if (stop) break;
+        it += ntile;
       }
       if (*abort_flag) {
         // let the copies already issued land before the CTA leaves
-        for (uint32_t u = (it > NST ? it - NST : 0); u < it; ++u) {
-          mbar_wait_drain(&sm.k_full[u % NST], (u / NST) & 1, kWait);
-          mbar_wait_drain(&sm.v_full[u % NST], (u / NST) & 1, kWait);
-        }
+        for (uint32_t u = (n_k > NKB ? n_k - NKB : 0); u < n_k; ++u)
+          mbar_wait_drain(&sm.k_full[u % NKB], (u / NKB) & 1, kWait);
+        for (uint32_t u = (n_v > NVB ? n_v - NVB : 0); u < n_v; ++u)
+          mbar_wait_drain(&sm.v_full[u % NVB], (u / NVB) & 1, kWait);
         if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
       }
     }
@@ -219,39 +235,47 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         int ntile = (t1 - t0 + BT - 1) / BT;
         if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
         tc_fence_after();
-        auto qk = [&](uint32_t g) -> bool {
-          int s = g % NST, b = g & 1;
-          if (!mbar_wait(&sm.k_full[s], (g / NST) & 1, kWait, abort_flag)) return false;
+        auto qk = [&](uint32_t g, int j) -> bool {
+          int s3 = g % NKB, b = g & 1;
+          if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag)) return false;
           if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
           tc_fence_after();
-          issue_qk(tm, sm.q, sm.k[s], b);
+          issue_qk(tm, sm.q, sm.k[s3], b);
           mma_commit(&sm.s_full[b]);
+          mma_commit(&sm.k_empty[s3]);
+          if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
           return true;
         };
-        if (ntile > 0) ok = qk(it);
+        if (ntile > 0) ok = qk(it, 0);
         // the O of the previous item must have been read out before P V overwrites it
         if (ok && n_local > 0 && !mbar_wait(&sm.o_empty, (n_local - 1) & 1, kWait, abort_flag)) ok = false;
         for (int j = 0; j < ntile && ok; ++j) {
           uint32_t g = it + j;
+          int s2 = g % NVB, b = g & 1;
+          // Q K^T of the next tile goes first when its operands are already there
+          bool next_issued = false;
           if (j + 1 < ntile) {
-            ok = qk(g + 1);
-            if (!ok) break;
-          } else {
-            mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
+            uint32_t g1 = g + 1;
+            if (mbar_try_wait(&sm.k_full[g1 % NKB], (g1 / NKB) & 1) &&
+                (g1 < 2 || mbar_try_wait(&sm.s_empty[g1 & 1], ((g1 >> 1) - 1) & 1))) {
+              ok = qk(g1, j + 1);
+              next_issued = true;
+              if (!ok) break;
+            }
           }
-          int s = g % NST, b = g & 1;
           if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
-              !mbar_wait(&sm.v_full[s], (g / NST) & 1, kWait, abort_flag)) {
+              !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
 #pragma unroll
-          for (int ks = 0; ks < BT / 16; ++ks) issue_pv_step(tm, 2 * BT, sm.v[s], b, ks, j == 0 && ks == 0);
+          for (int ks = 0; ks < BT / 16; ++ks) issue_pv_step(tm, 2 * BT, sm.v[s2], b, ks, j == 0 && ks == 0);
           mma_commit(&sm.s_empty[b]);
-          mma_commit(&sm.kv_empty[s]);
+          mma_commit(&sm.v_empty[s2]);
           mma_commit(&sm.pv_done);
           if (j + 1 == ntile) mma_commit(&sm.o_full);
+          if (ok && j + 1 < ntile && !next_issued) ok = qk(g + 1, j + 1);
         }
         it += ntile;
       }
