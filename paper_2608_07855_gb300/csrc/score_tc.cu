@@ -40,7 +40,7 @@ constexpr int NKB = 3;   // pass B: K stages (with their slot tables)
 constexpr int NVB = 2;   // pass B: V stages
 constexpr int SLOT = 16;
 constexpr int SLOTS = BT / SLOT;  // slots per pass-B tile
-constexpr int NFIFO = 8;          // page-sum FIFO depth (>= SLOTS)
+constexpr int NFIFO = 16;         // page-sum FIFO depth (>= 2 x SLOTS)
 constexpr uint64_t kWait = 1000000000ull;
 constexpr float kLazy = 8.0f;     // rescale O when the max grows by > 2^8
 
@@ -252,17 +252,9 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         for (int j = 0; j < ntile && ok; ++j) {
           uint32_t g = it + j;
           int s2 = g % NVB, b = g & 1;
-          // Q K^T of the next tile goes first when its operands are already there
-          bool next_issued = false;
-          if (j + 1 < ntile) {
-            uint32_t g1 = g + 1;
-            if (mbar_try_wait(&sm.k_full[g1 % NKB], (g1 / NKB) & 1) &&
-                (g1 < 2 || mbar_try_wait(&sm.s_empty[g1 & 1], ((g1 >> 1) - 1) & 1))) {
-              ok = qk(g1, j + 1);
-              next_issued = true;
-              if (!ok) break;
-            }
-          }
+          // Q K^T of the next tile first, so that it runs while the softmax
+          // works on this one (its K is prefetched three tiles deep)
+          if (j + 1 < ntile && !(ok = qk(g + 1, j + 1))) break;
           if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
               !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
             ok = false;
@@ -275,7 +267,6 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
           mma_commit(&sm.v_empty[s2]);
           mma_commit(&sm.pv_done);
           if (j + 1 == ntile) mma_commit(&sm.o_full);
-          if (ok && j + 1 < ntile && !next_issued) ok = qk(g + 1, j + 1);
         }
         it += ntile;
       }
@@ -577,19 +568,16 @@ struct SmemB {
   SlotMeta meta[NKB][SLOTS];
   int page_of[NKB][SLOTS];  // page id of each slot
   uint32_t tile_bytes[NKB]; // bytes of the tile's K (and V) copies
+  int tile_full[NKB];       // every slot of the tile lies in the prefix all probe rows see
   int pos[4][BT];           // per softmax warp: positions of the current tile
   int pg_start[kSlotsPerItem];  // the producer's copy of the item's page table
   int pg_len[kSlotsPerItem];
   int pg_slots[kSlotsPerItem];
-  float red[2][BM];         // per page parity: the upper channel half of ||U - S o||^2
-  float ssum[SLOTS][BM];    // per softmax thread: slot sums of the current tile
-  int scnt[SLOTS][BM];      // and visible counts
   float fifo_s[NFIFO][BM];  // per page: S_E of every row
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
   uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], meta_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2],
-      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], red_full[2],
-      red_empty[2], drain;
+      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain;
   uint32_t tmem;
   int abort_flag;
 };
@@ -646,14 +634,12 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       mbar_init(&sm.s_full[b], 1);
       mbar_init(&sm.s_empty[b], 1);
       mbar_init(&sm.acc_full[b], 1);
-      mbar_init(&sm.acc_empty[b], 8);
-      mbar_init(&sm.red_full[b], 4);
-      mbar_init(&sm.red_empty[b], 4);
+      mbar_init(&sm.acc_empty[b], 4);  // the epilogue warpgroup of that page parity
     }
     mbar_init(&sm.p_full, 4);
     for (int f = 0; f < NFIFO; ++f) {
       mbar_init(&sm.fifo_full[f], 4);
-      mbar_init(&sm.fifo_empty[f], 8);
+      mbar_init(&sm.fifo_empty[f], 4);
     }
     mbar_init(&sm.drain, 1);
     fence_mbar_init();
@@ -669,9 +655,10 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
 
   // warpgroup 0: TMA producer, MMA issuer and two idle warps; 1: softmax;
   // 2 and 3: epilogue.  Each branch first sets its warpgroup's register
-  // budget: 56 + 136 + 2 x 160 per thread = the launch's 4 x 128.
+  // budget: 64 + 112 + 2 x 168 per thread = the launch's 4 x 128 (a budget
+  // below 128 is set with a decrease, above it with an increase).
   if (warp < 4) {
-    regs_dec<56>();  // warps 2 and 3 stay idle
+    regs_dec<64>();  // warps 2 and 3 stay idle
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
       // The whole warp copies each item's page table into shared memory; lane 0
@@ -711,6 +698,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             };
             int e = 0, sub = 0;
             while (e < np && pslots(e) == 0) ++e;
+            const int vis_all = tr.prep->vis_all;
             // runs of slots whose rows are contiguous in memory (full pages of
             // one event) travel as one box of 16, 32, 64 or 128 rows
             auto issue_boxes = [&](int s3, uint8_t *dst, const CUtensorMap *big, const CUtensorMap *small,
@@ -749,6 +737,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                                !mbar_wait(&sm.meta_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)))
                 return false;
               uint32_t bytes = 0;
+              int tfull = 1;
 #pragma unroll 1
               for (int q = 0; q < SLOTS; ++q) {
                 SlotMeta mt;
@@ -758,6 +747,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                   mt.nv = min(SLOT, pl - sub * SLOT);
                   mt.po = po;
                   mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
+                  tfull &= mt.tok0 + mt.nv <= vis_all;
                   sm.page_of[s3][q] = bi.E0 + e;
                   bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
                   if (++sub * SLOT >= pl) {
@@ -776,6 +766,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
                 sm.meta[s3][q] = mt;
               }
               sm.tile_bytes[s3] = bytes;
+              sm.tile_full[s3] = tfull;
               // the slot table is written before the arrival that publishes it
               mbar_expect_tx(&sm.k_full[s3], bytes);
               issue_boxes(s3, sm.k[s3], &mp.k, mp.kb, &sm.k_full[s3]);
@@ -839,17 +830,9 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           for (int j = 0; j < ntile && ok; ++j) {
             uint32_t g = it + j;
             int s3 = g % NKB, s2 = g % NVB, b = g & 1;
-            // Q K^T of the next tile goes first when its operands are already there
-            bool next_issued = false;
-            if (j + 1 < ntile) {
-              uint32_t g1 = g + 1;
-              if (mbar_try_wait(&sm.k_full[g1 % NKB], (g1 / NKB) & 1) &&
-                  (g1 < 2 || mbar_try_wait(&sm.s_empty[g1 & 1], ((g1 >> 1) - 1) & 1))) {
-                ok = qk(g1, j + 1);
-                next_issued = true;
-                if (!ok) break;
-              }
-            }
+            // Q K^T of the next tile first, so that it runs while the softmax
+            // works on this one (its K is prefetched three tiles deep)
+            if (j + 1 < ntile && !(ok = qk(g + 1, j + 1))) break;
             if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
                 !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
               ok = false;
@@ -874,7 +857,6 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             mma_commit(&sm.s_empty[b]);
             mma_commit(&sm.v_empty[s2]);
             mbar_arrive(&sm.meta_empty[s3]);  // done with the slot table
-            if (ok && j + 1 < ntile && !next_issued) ok = qk(g + 1, j + 1);
           }
           it += ntile;
         }
@@ -886,7 +868,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     }
   } else if (warp < 8) {
     // ------------------------------------------------------------ softmax (warps 4..7)
-    regs_inc<136>();
+    regs_dec<112>();  // below the launch's 128: a decrease
     const int wq = warp & 3;
     const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
@@ -911,7 +893,6 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         float mn = tr.stats[(((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4)];
         if (mn != -INFINITY) neg_m2 = -mn * 1.4426950408889634f;
       }
-      const int vis_all = tr.prep->vis_all;
       int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
       for (int j = 0; j < ntile && ok; ++j) {
         uint32_t g = it + j;
@@ -922,12 +903,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           break;
         }
         // slots inside the prefix every probe row sees need no position test
-        bool full = true;
-#pragma unroll 1
-        for (int q = 0; q < SLOTS; ++q) {
-          const SlotMeta mt = sm.meta[s][q];
-          full &= mt.po < 0 || mt.tok0 + mt.nv <= vis_all;
-        }
+        const bool full = sm.tile_full[s] != 0;
         if (!full) {  // each warp keeps its own copy: no cross-warp barrier
           __syncwarp();
 #pragma unroll 1
@@ -945,16 +921,18 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         tc_fence_after();
         // Per 32-column chunk (two slots): e = exp(s - m) on the visible page
         // tokens (a visibility bit mask turns the others into -inf, so e = 0);
-        // per-slot sums and counts to shared memory; P as the (hi, lo) bf16
-        // pair written over the S columns just read.  The chunk loop is not
-        // unrolled: a small loop body keeps the instruction cache warm.
+        // P as the (hi, lo) bf16 pair written over the S columns just read;
+        // slot sums accumulate into page sums S_E, which go to the page FIFO
+        // when the page's last slot is done.  The chunk loop is not unrolled:
+        // a small loop body keeps the instruction cache warm.
+        const int po_first = po_seen;
 #pragma unroll 1
-        for (int ch = 0; ch < BT / 32; ++ch) {
+        for (int ch = 0; ch < BT / 32 && ok; ++ch) {
           float x[32];
           tmem_ld32f(tm + lane_base + b * BT + 32 * ch, x);
-          const int nv0 = sm.meta[s][2 * ch].nv, nv1 = sm.meta[s][2 * ch + 1].nv;
-          uint32_t vm = (nv0 >= SLOT ? 0xffffu : (1u << max(nv0, 0)) - 1u) |
-                        ((nv1 >= SLOT ? 0xffffu : (1u << max(nv1, 0)) - 1u) << 16);
+          const SlotMeta m0 = sm.meta[s][2 * ch], m1 = sm.meta[s][2 * ch + 1];
+          uint32_t vm = (m0.nv >= SLOT ? 0xffffu : (1u << max(m0.nv, 0)) - 1u) |
+                        ((m1.nv >= SLOT ? 0xffffu : (1u << max(m1.nv, 0)) - 1u) << 16);
           if (!full) {
 #pragma unroll 1
             for (int i = 0; i < 32; ++i)
@@ -975,43 +953,40 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             c0 += x[16 + i];
             c1 += x[17 + i];
           }
-          sm.ssum[2 * ch][row] = a0 + a1;
-          sm.ssum[2 * ch + 1][row] = c0 + c1;
-          sm.scnt[2 * ch][row] = __popc(vm & 0xffffu);
-          sm.scnt[2 * ch + 1][row] = __popc(vm >> 16);
           uint32_t pk[32];
           split_pack32(x, pk);
           tmem_st32(tm + lane_base + b * BT + 32 * ch, pk);
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const SlotMeta mt = h2 ? m1 : m0;
+            if (mt.po < 0) continue;
+            if (mt.flags & 1) {
+              S_cur = 0.0f;
+              n_cur = 0;
+            }
+            S_cur += h2 ? c0 + c1 : a0 + a1;
+            n_cur += __popc(h2 ? vm >> 16 : vm & 0xffffu);
+            if (mt.flags & 2) {
+              int f = po_seen % NFIFO;
+              if (po_seen >= NFIFO &&
+                  !mbar_wait(&sm.fifo_empty[f], ((po_seen / NFIFO) - 1) & 1, kWait, abort_flag)) {
+                ok = false;
+                break;
+              }
+              sm.fifo_s[f][row] = S_cur;
+              sm.fifo_n[f][row] = n_cur;
+              if (row == 0) sm.fifo_page[f] = sm.page_of[s][2 * ch + h2];
+              ++po_seen;
+            }
+          }
         }
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_full);
-        // page sums: walk the slots in order, hand finished pages to the epilogue
-#pragma unroll 1
-        for (int q = 0; q < SLOTS; ++q) {
-          const SlotMeta mt = sm.meta[s][q];
-          if (mt.po < 0 || !ok) continue;
-          if (mt.flags & 1) {
-            S_cur = 0.0f;
-            n_cur = 0;
-          }
-          S_cur += sm.ssum[q][row];
-          n_cur += sm.scnt[q][row];
-          if (mt.flags & 2) {
-            int f = po_seen % NFIFO;
-            if (po_seen >= NFIFO &&
-                !mbar_wait(&sm.fifo_empty[f], ((po_seen / NFIFO) - 1) & 1, kWait, abort_flag)) {
-              ok = false;
-              continue;
-            }
-            sm.fifo_s[f][row] = S_cur;
-            sm.fifo_n[f][row] = n_cur;
-            if (row == 0) sm.fifo_page[f] = sm.page_of[s][q];
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.fifo_full[f]);
-            ++po_seen;
-          }
+        if (lane == 0) {
+          mbar_arrive(&sm.p_full);
+          // publish the pages this tile finished to the epilogue
+          for (int k = po_first; k < po_seen; ++k) mbar_arrive(&sm.fifo_full[k % NFIFO]);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.meta_empty[s]);  // done with the slot table
@@ -1020,14 +995,15 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     }
   } else {
     // ------------------------------------------------------------ epilogue (warps 8..15)
-    // Two warpgroups split the 128 channels; each thread owns one row and 64
-    // channels of that row's output o.
-    regs_inc<160>();
+    // The two warpgroups take alternate pages: warpgroup 2 the even page
+    // ordinals (accumulator U[0]), warpgroup 3 the odd ones (U[1]).  Each
+    // thread owns one row and all 128 channels of that row's output o.
+    regs_inc<168>();
     const int wq = warp & 3;
-    const int half = (warp - 8) >> 2;
+    const int par = (warp - 8) >> 2;
     const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
-    constexpr int DH = D / 2;
+    const uint32_t u_col = 2 * BT + par * D;
     int po = 0;
     bool ok = true;
     for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
@@ -1038,7 +1014,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       int grow = bi.rt * BM + row;
       bool valid_row = grow < rows;
       int h = bi.kvh * L.g + (valid_row ? grow / tr.W : 0), w = valid_row ? grow % tr.W : 0;
-      float2 o2[DH / 2];
+      float2 o2[D / 2];
       float lsum = 0.0f, onorm = 0.0f;
       int nvis = 0;
       {
@@ -1051,18 +1027,17 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         for (int c = 0; c < D; c += 4) {
           float4 v = valid_row ? *reinterpret_cast<const float4 *>(st + 4 + c) : make_float4(0.f, 0.f, 0.f, 0.f);
           ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-          if ((c >> 6) == half) {
-            o2[(c & 63) / 2] = make_float2(v.x, v.y);
-            o2[(c & 63) / 2 + 1] = make_float2(v.z, v.w);
-          }
+          o2[c / 2] = make_float2(v.x, v.y);
+          o2[c / 2 + 1] = make_float2(v.z, v.w);
         }
         onorm = sqrtf(ss);
       }
       int npages = tr.items[2 * bi.k + 1].x;
       for (int k = 0; k < npages && ok; ++k, ++po) {
-        int a = po & 1, f = po % NFIFO;
+        if ((po & 1) != par) continue;
+        int f = po % NFIFO;
         if (!mbar_wait(&sm.fifo_full[f], (po / NFIFO) & 1, kWait, abort_flag) ||
-            !mbar_wait(&sm.acc_full[a], (po >> 1) & 1, kWait, abort_flag)) {
+            !mbar_wait(&sm.acc_full[par], (po >> 1) & 1, kWait, abort_flag)) {
           ok = false;
           break;
         }
@@ -1071,55 +1046,36 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         int n_E = sm.fifo_n[f][row];
         int E = sm.fifo_page[f];
         const float2 nS = make_float2(-S_E, -S_E);
-        // copy this half of U_E out of TMEM, then hand the accumulator back
-        uint32_t r0[32], r1[32];
-        tmem_ld64(tm + lane_base + 2 * BT + a * D + half * DH, r0, r1);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&sm.acc_empty[a]);
-          mbar_arrive(&sm.fifo_empty[f]);
-        }
+        // ||U_E - S_E o||^2 over 16-column pieces of U_E
         float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-          float2 d0 = ffma2(nS, o2[i / 2], make_float2(__uint_as_float(r0[i]), __uint_as_float(r0[i + 1])));
-          float2 d1 = ffma2(nS, o2[i / 2 + 1], make_float2(__uint_as_float(r0[i + 2]), __uint_as_float(r0[i + 3])));
-          acc0 = ffma2(d0, d0, acc0);
-          acc1 = ffma2(d1, d1, acc1);
-        }
-#pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-          float2 d0 = ffma2(nS, o2[16 + i / 2], make_float2(__uint_as_float(r1[i]), __uint_as_float(r1[i + 1])));
-          float2 d1 = ffma2(nS, o2[16 + i / 2 + 1], make_float2(__uint_as_float(r1[i + 2]), __uint_as_float(r1[i + 3])));
-          acc0 = ffma2(d0, d0, acc0);
-          acc1 = ffma2(d1, d1, acc1);
-        }
-        float part = (acc0.x + acc0.y) + (acc1.x + acc1.y);
-        const int pb = po & 1;
-        if (half == 1) {  // hand the upper half to the lower warpgroup
-          if (po >= 2 && !mbar_wait(&sm.red_empty[pb], ((po >> 1) - 1) & 1, kWait, abort_flag)) {
-            ok = false;
-            break;
+        for (int c0 = 0; c0 < D; c0 += 16) {
+          uint32_t r[16];
+          tmem_ld16(tm + lane_base + u_col + c0, r);
+          tmem_wait_ld();
+          if (c0 + 16 == D) {  // U_E is in registers: hand the accumulator back
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+              mbar_arrive(&sm.acc_empty[par]);
+              mbar_arrive(&sm.fifo_empty[f]);
+            }
           }
-          sm.red[pb][row] = part;
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.red_full[pb]);
-        } else {
-          if (!mbar_wait(&sm.red_full[pb], (po >> 1) & 1, kWait, abort_flag)) {
-            ok = false;
-            break;
-          }
-          float num2 = part + sm.red[pb][row];
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.red_empty[pb]);
-          float r = valid_row ? effect_value(n_E, nvis, S_E, lsum, num2, onorm) : 0.0f;
-          if (valid_row && tr.headR) atomic_max_nonneg(tr.headR + ((int64_t)bi.l * L.Hq + h) * tr.P + E, r);
-          float rm = r;
 #pragma unroll
-          for (int off = 16; off > 0; off >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, off));
-          if (lane == 0) atomic_max_nonneg(tr.R + E, rm);
+          for (int i = 0; i < 16; i += 4) {
+            float2 d0 = ffma2(nS, o2[(c0 + i) / 2], make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])));
+            float2 d1 = ffma2(nS, o2[(c0 + i) / 2 + 1], make_float2(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])));
+            acc0 = ffma2(d0, d0, acc0);
+            acc1 = ffma2(d1, d1, acc1);
+          }
         }
+        float num2 = (acc0.x + acc0.y) + (acc1.x + acc1.y);
+        float r = valid_row ? effect_value(n_E, nvis, S_E, lsum, num2, onorm) : 0.0f;
+        if (valid_row && tr.headR) atomic_max_nonneg(tr.headR + ((int64_t)bi.l * L.Hq + h) * tr.P + E, r);
+        float rm = r;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, off));
+        if (lane == 0) atomic_max_nonneg(tr.R + E, rm);
       }
     }
   }
