@@ -159,7 +159,8 @@ size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *
   for (int t = 0; t < n_traj; ++t) {
     TcCounts c = tc_counts(s, tr[t], tc_chunk_len(1, &tr[t]));
     items += (size_t)s->layers * s->kv_heads * tc_chunk_bound(tr[t].S) * c.nrt;
-    slots += align_up((size_t)(tr[t].P + 1) * 4) + align_up((size_t)c.nbitem * 32) + kAlign;
+    slots += align_up((size_t)(tr[t].P + 1) * 4) + align_up((size_t)c.nbitem * 32) + kAlign +
+             align_up(((size_t)cdiv(tr[t].S, 16) + tr[t].P) * 16);
   }
   return align_up(items * tc::kRowsPerTile * 132 * 4) + slots;
 }
@@ -376,6 +377,8 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
       slot_base += align_up((size_t)c.nbitem * 32);
       tt.prep = reinterpret_cast<tc::TcPrep *>(slot_base);
       slot_base += kAlign;
+      tt.slot_tab = reinterpret_cast<int4 *>(slot_base);
+      slot_base += align_up(((size_t)cdiv(x.S, 16) + x.P) * 16);
       tt.stats = L.stats[t];
       tt.R = L.R[t];
       tt.headR = L.headR[t];

@@ -35,7 +35,6 @@ using namespace ckv::sm103;
 constexpr int D = 128;
 constexpr int BM = 128;  // probe rows per tile (MMA M)
 constexpr int BT = 128;  // KV rows per tile (MMA N of Q K^T, K of P V)
-constexpr int NST = 2;   // K/V pipeline stages (pass A)
 constexpr int NKB = 3;   // pass B: K stages (with their slot tables)
 constexpr int NVB = 2;   // pass B: V stages
 constexpr int SLOT = 16;
@@ -469,51 +468,63 @@ __global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaun
 // Per trajectory, once per call:
 //   slot_off[E] = sum over F < E of ceil(len_F / 16), slot_off[P] = total
 //   (a page that fails the table checks gets no slot and an error is recorded);
+//   slot_tab[slot] = {first token, valid tokens, page, first/last flags and
+//   the page's rank among the pages with slots} for every 16-token slot;
 //   the pass-B work items: item k takes the pages whose first slot lies in
 //   [k * slots_per_item, (k + 1) * slots_per_item);
 //   vis_all = number of leading resident tokens visible to every probe row
 //   (positions increase, so this is a prefix).
 __global__ void __launch_bounds__(1024) prep_kernel(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   const TcTraj &tr = L.t[blockIdx.x];
-  __shared__ int s_warp[32];
-  __shared__ int s_base;
-  if (threadIdx.x == 0) s_base = 0;
-  __syncthreads();
   int lane = threadIdx.x % 32, wid = threadIdx.x / 32;
+  // one scan gives both the slot offsets (low 32 bits) and the rank of each
+  // page among the pages that have slots (high 32 bits)
+  __shared__ unsigned long long s_w64[32];
+  __shared__ unsigned long long s_b64;
+  if (threadIdx.x == 0) s_b64 = 0ull;
+  __syncthreads();
   for (int c0 = 0; c0 < tr.P; c0 += 1024) {
     int E = c0 + threadIdx.x;
-    int v = 0;
+    int ns = 0, ps = 0, pl = 0;
     if (E < tr.P) {
-      int ps = tr.ps[E], pl = tr.pl[E];
+      ps = tr.ps[E];
+      pl = tr.pl[E];
       bool bad = pl < 0 || ps < 0 || ps > tr.S - pl || (E > 0 && ps < tr.ps[E - 1] + tr.pl[E - 1]);
       if (bad) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, E);
-      v = bad ? 0 : (pl + SLOT - 1) / SLOT;
+      ns = bad ? 0 : (pl + SLOT - 1) / SLOT;
     }
-    int x = v;
+    const unsigned long long v = ((unsigned long long)(ns > 0) << 32) | (unsigned)ns;
+    unsigned long long x = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int y = __shfl_up_sync(0xffffffffu, x, o);
+      unsigned long long y = __shfl_up_sync(0xffffffffu, x, o);
       if (lane >= o) x += y;
     }
-    if (lane == 31) s_warp[wid] = x;
+    if (lane == 31) s_w64[wid] = x;
     __syncthreads();
     if (wid == 0) {
-      int w = s_warp[lane];
+      unsigned long long w = s_w64[lane];
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        int y = __shfl_up_sync(0xffffffffu, w, o);
+        unsigned long long y = __shfl_up_sync(0xffffffffu, w, o);
         if (lane >= o) w += y;
       }
-      s_warp[lane] = w;
+      s_w64[lane] = w;
     }
     __syncthreads();
-    int excl = s_base + (wid ? s_warp[wid - 1] : 0) + x - v;
-    if (E < tr.P) tr.slot_off[E] = excl;
+    const unsigned long long excl = s_b64 + (wid ? s_w64[wid - 1] : 0ull) + x - v;
+    if (E < tr.P) {
+      const int off = (int)(excl & 0xffffffffull), rank = (int)(excl >> 32);
+      tr.slot_off[E] = off;
+      for (int sub = 0; sub < ns; ++sub)
+        tr.slot_tab[off + sub] = make_int4(ps + sub * SLOT, min(SLOT, pl - sub * SLOT), E,
+                                           (sub == 0 ? 1 : 0) | (sub + 1 == ns ? 2 : 0) | (rank << 2));
+    }
     __syncthreads();
-    if (threadIdx.x == 0) s_base += s_warp[31];
+    if (threadIdx.x == 0) s_b64 += s_w64[31];
     __syncthreads();
   }
-  if (threadIdx.x == 0) tr.slot_off[tr.P] = s_base;
+  if (threadIdx.x == 0) tr.slot_off[tr.P] = (int)(s_b64 & 0xffffffffull);
   __syncthreads();
   for (int k = threadIdx.x; k < tr.nbitem; k += 1024) {
     int lo = k * L.slots_per_item, hi = lo + L.slots_per_item;
@@ -570,9 +581,6 @@ struct SmemB {
   uint32_t tile_bytes[NKB]; // bytes of the tile's K (and V) copies
   int tile_full[NKB];       // every slot of the tile lies in the prefix all probe rows see
   int pos[4][BT];           // per softmax warp: positions of the current tile
-  int pg_start[kSlotsPerItem];  // the producer's copy of the item's page table
-  int pg_len[kSlotsPerItem];
-  int pg_slots[kSlotsPerItem];
   float fifo_s[NFIFO][BM];  // per page: S_E of every row
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
@@ -607,8 +615,6 @@ __device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
   b.nslot = e.w;
   return b;
 }
-
-__device__ __forceinline__ bool has_slots(const TcTraj &tr, int E) { return tr.slot_off[E + 1] > tr.slot_off[E]; }
 
 __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   extern __shared__ uint8_t smem_raw[];
@@ -661,11 +667,12 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     regs_dec<64>();  // warps 2 and 3 stay idle
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
-      // The whole warp copies each item's page table into shared memory; lane 0
-      // then walks the slots and issues the copies.
+      // The whole warp works each tile: lanes 0..7 take one 16-token slot each
+      // from the slot table, write the tile's slot table to shared memory and
+      // issue the copies of the runs of slots that start at them.
       uint64_t pol = policy_evict_first();
       uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
-      int po = 0;  // page ordinal
+      int po_base = 0;  // page ordinal of the item's first page
       bool stop = false;
       for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
         if (*abort_flag) break;
@@ -673,127 +680,101 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         if (bi.nslot == 0) continue;
         const TcTraj &tr = L.t[bi.t];
         const TcMaps &mp = L.maps[bi.t];
-        // pages of the item; zero-length pages take no slot, so there may be more
-        // pages than the copy holds: those are read from global memory
-        int np = bi.E1 - bi.E0;
-        for (int e = lane; e < min(np, kSlotsPerItem); e += 32) {
-          int E = bi.E0 + e;
-          sm.pg_start[e] = tr.ps[E];
-          sm.pg_len[e] = tr.pl[E];
-          sm.pg_slots[e] = tr.slot_off[E + 1] - tr.slot_off[E];
+        const int4 *stab = tr.slot_tab + bi.slot0;
+        const int rank0 = stab[0].w >> 2;  // slotted-page rank of the item's first page
+        const int vis_all = tr.prep->vis_all;
+        if (n_local > 0 && !__all_sync(0xffffffffu, mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag))) {
+          stop = true;
+          break;
         }
-        __syncwarp();
         if (lane == 0) {
-          if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) {
-            stop = true;
-          } else {
-            mbar_expect_tx(&sm.q_full, kTileBytes);
-            int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
-            tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
-            tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
-            ++n_local;
-            // page cursor; pages without slots (empty or rejected by the slot scan) are skipped
-            auto pslots = [&](int e) {
-              return e < kSlotsPerItem ? sm.pg_slots[e] : tr.slot_off[bi.E0 + e + 1] - tr.slot_off[bi.E0 + e];
-            };
-            int e = 0, sub = 0;
-            while (e < np && pslots(e) == 0) ++e;
-            const int vis_all = tr.prep->vis_all;
-            // runs of slots whose rows are contiguous in memory (full pages of
-            // one event) travel as one box of 16, 32, 64 or 128 rows
-            auto issue_boxes = [&](int s3, uint8_t *dst, const CUtensorMap *big, const CUtensorMap *small,
-                                   uint64_t *bar) {
-              int q = 0;
-              while (q < SLOTS) {
-                const SlotMeta m0 = sm.meta[s3][q];
-                if (m0.po < 0) {
-                  ++q;
-                  continue;
-                }
-                int run = 1;
-                while (q + run < SLOTS && sm.meta[s3][q + run].po >= 0 &&
-                       sm.meta[s3][q + run].tok0 == m0.tok0 + run * SLOT && sm.meta[s3][q + run - 1].nv == SLOT)
-                  ++run;
-                int done = 0;
-                while (done < run) {
-                  int rem = run - done;
-                  int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
-                  if (lg == 3 && (q + done) != 0) lg = 2;  // a 128-row box covers the whole tile
-                  int tok = m0.tok0 + done * SLOT;
-                  uint8_t *d = dst + (q + done) * SLOT * 128;
-                  const CUtensorMap *m = lg == 3 ? big : small + lg;
-                  tma4(d, m, 0, tok, bi.kvh, bi.l, bar, pol);
-                  tma4(d + kHalf, m, 64, tok, bi.kvh, bi.l, bar, pol);
-                  done += 1 << lg;
-                }
-                q += run;
-              }
-            };
-            // K of tile g (and its slot table) once Q K^T of tile g - 3 is done and
-            // its slot table released
-            auto load_k = [&](uint32_t g) -> bool {
-              int s3 = g % NKB;
-              if (g >= NKB && (!mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag) ||
-                               !mbar_wait(&sm.meta_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)))
-                return false;
-              uint32_t bytes = 0;
-              int tfull = 1;
-#pragma unroll 1
-              for (int q = 0; q < SLOTS; ++q) {
-                SlotMeta mt;
-                if (e < np) {
-                  int pl = e < kSlotsPerItem ? sm.pg_len[e] : tr.pl[bi.E0 + e];
-                  mt.tok0 = (e < kSlotsPerItem ? sm.pg_start[e] : tr.ps[bi.E0 + e]) + sub * SLOT;
-                  mt.nv = min(SLOT, pl - sub * SLOT);
-                  mt.po = po;
-                  mt.flags = (sub == 0 ? 1 : 0) | ((sub + 1) * SLOT >= pl ? 2 : 0);
-                  tfull &= mt.tok0 + mt.nv <= vis_all;
-                  sm.page_of[s3][q] = bi.E0 + e;
-                  bytes += 2 * SLOT * 128;  // two 64-channel boxes of 16 rows
-                  if (++sub * SLOT >= pl) {
-                    sub = 0;
-                    ++po;
-                    ++e;
-                    while (e < np && pslots(e) == 0) ++e;
-                  }
-                } else {
-                  mt.tok0 = 0;
-                  mt.nv = 0;
-                  mt.po = -1;
-                  mt.flags = 0;
-                  sm.page_of[s3][q] = -1;
-                }
-                sm.meta[s3][q] = mt;
-              }
-              sm.tile_bytes[s3] = bytes;
-              sm.tile_full[s3] = tfull;
-              // the slot table is written before the arrival that publishes it
-              mbar_expect_tx(&sm.k_full[s3], bytes);
-              issue_boxes(s3, sm.k[s3], &mp.k, mp.kb, &sm.k_full[s3]);
-              ++n_k;
-              return true;
-            };
-            // V of tile g once P V of tile g - 2 is done
-            auto load_v = [&](uint32_t g) -> bool {
-              int s3 = g % NKB, s2 = g % NVB;
-              if (g >= NVB && !mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag)) return false;
-              mbar_expect_tx(&sm.v_full[s2], sm.tile_bytes[s3]);
-              issue_boxes(s3, sm.v[s2], &mp.v, mp.vb, &sm.v_full[s2]);
-              ++n_v;
-              return true;
-            };
-            // K runs one tile ahead of V
-            int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-            stop = !load_k(it);
-            for (int j = 0; j < ntile && !stop; ++j) {
-              if (j + 1 < ntile && !load_k(it + j + 1)) stop = true;
-              else if (!load_v(it + j)) stop = true;
-            }
-            it += ntile;
-          }
+          mbar_expect_tx(&sm.q_full, kTileBytes);
+          int qrow = (bi.l * L.Hq + bi.kvh * L.g) * tr.W + bi.rt * BM;
+          tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+          tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
         }
-        stop = __shfl_sync(0xffffffffu, stop, 0);
-        __syncwarp();
+        ++n_local;
+        // Copies of the runs of slots whose rows are contiguous in memory (full
+        // slots of one event): a lane that starts a run issues its boxes of 16,
+        // 32, 64 or 128 rows.  Called by the whole warp; lanes 0..7 carry a slot.
+        auto issue_runs = [&](int tok0, int nv, bool valid, uint8_t *dst, const CUtensorMap *big,
+                              const CUtensorMap *small, uint64_t *bar) {
+          unsigned vmask = __ballot_sync(0xffffffffu, valid);
+          int ptok = __shfl_up_sync(0xffffffffu, tok0, 1), pnv = __shfl_up_sync(0xffffffffu, nv, 1);
+          bool pvalid = lane > 0 && ((vmask >> (lane - 1)) & 1u);
+          bool start = valid && (!pvalid || pnv != SLOT || ptok + SLOT != tok0);
+          unsigned smask = __ballot_sync(0xffffffffu, start);
+          if (start) {
+            unsigned ends = (smask | ~vmask) & ~((2u << lane) - 1u);  // run boundaries after this lane
+            int run = (__ffs(ends) - 1) - lane;                        // lanes >= 8 are never valid
+            int done = 0;
+            while (done < run) {
+              int rem = run - done;
+              int lg = rem >= 8 ? 3 : rem >= 4 ? 2 : rem >= 2 ? 1 : 0;
+              if (lg == 3 && (lane + done) != 0) lg = 2;  // a 128-row box covers the whole tile
+              int tok = tok0 + done * SLOT;
+              uint8_t *d = dst + (lane + done) * SLOT * 128;
+              const CUtensorMap *m = lg == 3 ? big : small + lg;
+              tma4(d, m, 0, tok, bi.kvh, bi.l, bar, pol);
+              tma4(d + kHalf, m, 64, tok, bi.kvh, bi.l, bar, pol);
+              done += 1 << lg;
+            }
+          }
+        };
+        // K of tile g (and its slot table) once Q K^T of tile g - 3 is done and
+        // its slot table released
+        auto load_k = [&](uint32_t g, int j) -> bool {
+          int s3 = g % NKB;
+          bool w_ok = g < NKB || (mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag) &&
+                                  mbar_wait(&sm.meta_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag));
+          if (!__all_sync(0xffffffffu, w_ok)) return false;
+          int sl = j * SLOTS + lane;
+          bool valid = lane < SLOTS && sl < bi.nslot;
+          int4 rec = valid ? stab[sl] : make_int4(0, 0, -1, 0);
+          SlotMeta mt;
+          mt.tok0 = rec.x;
+          mt.nv = valid ? rec.y : 0;
+          mt.po = valid ? po_base + (rec.w >> 2) - rank0 : -1;
+          mt.flags = valid ? rec.w & 3 : 0;
+          if (lane < SLOTS) {
+            sm.meta[s3][lane] = mt;
+            sm.page_of[s3][lane] = rec.z;
+          }
+          const bool tfull = __all_sync(0xffffffffu, !valid || rec.x + rec.y <= vis_all);
+          const uint32_t bytes = __popc(__ballot_sync(0xffffffffu, valid)) * 2u * SLOT * 128u;
+          __syncwarp();  // the slot table is written before the arrival that publishes it
+          if (lane == 0) {
+            sm.tile_bytes[s3] = bytes;
+            sm.tile_full[s3] = tfull;
+            mbar_expect_tx(&sm.k_full[s3], bytes);
+          }
+          __syncwarp();
+          issue_runs(mt.tok0, mt.nv, valid, sm.k[s3], &mp.k, mp.kb, &sm.k_full[s3]);
+          ++n_k;
+          return true;
+        };
+        // V of tile g once P V of tile g - 2 is done
+        auto load_v = [&](uint32_t g) -> bool {
+          int s3 = g % NKB, s2 = g % NVB;
+          bool w_ok = g < NVB || mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag);
+          if (!__all_sync(0xffffffffu, w_ok)) return false;
+          SlotMeta mt = sm.meta[s3][lane < SLOTS ? lane : 0];
+          bool valid = lane < SLOTS && mt.po >= 0;
+          if (lane == 0) mbar_expect_tx(&sm.v_full[s2], sm.tile_bytes[s3]);
+          __syncwarp();
+          issue_runs(mt.tok0, mt.nv, valid, sm.v[s2], &mp.v, mp.vb, &sm.v_full[s2]);
+          ++n_v;
+          return true;
+        };
+        // K runs one tile ahead of V
+        int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+        stop = !load_k(it, 0);
+        for (int j = 0; j < ntile && !stop; ++j) {
+          if (j + 1 < ntile && !load_k(it + j + 1, j + 1)) stop = true;
+          else if (!load_v(it + j)) stop = true;
+        }
+        it += ntile;
+        po_base += tr.items[2 * bi.k + 1].x;
       }
       if (lane == 0 && *abort_flag) {
         // let the copies already issued land before the CTA leaves

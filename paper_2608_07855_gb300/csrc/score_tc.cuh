@@ -28,6 +28,7 @@ struct TcTraj {
   const int32_t *pos, *qpos, *ps, *pl;
   int32_t *slot_off;  // workspace [P + 1]
   int4 *items;        // workspace [nbitem][2]: {E0, E1, slot0, nslot}, {npages, 0, 0, 0}
+  int4 *slot_tab;     // workspace [ceil(S/16) + P]: {tok0, nv, page, first | last << 1 | rank << 2}
   TcPrep *prep;       // workspace
   float *stats;       // [M][Hq][W][132]
   float *R;           // [P]
