@@ -585,7 +585,7 @@ struct SmemB {
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
   uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], meta_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2],
-      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain;
+      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain, drain2;
   uint32_t tmem;
   int abort_flag;
 };
@@ -648,6 +648,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       mbar_init(&sm.fifo_empty[f], 4);
     }
     mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain2, 1);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -659,12 +660,12 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
   tc_fence_after();
   const uint32_t tm = sm.tmem;
 
-  // warpgroup 0: TMA producer, MMA issuer and two idle warps; 1: softmax;
+  // warpgroup 0: TMA producer, P V issuer, Q K^T issuer, one idle warp; 1: softmax;
   // 2 and 3: epilogue.  Each branch first sets its warpgroup's register
   // budget: 64 + 112 + 2 x 168 per thread = the launch's 4 x 128 (a budget
   // below 128 is set with a decrease, above it with an increase).
   if (warp < 4) {
-    regs_dec<64>();  // warps 2 and 3 stay idle
+    regs_dec<64>();  // warp 3 stays idle
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
       // The whole warp works each tile: lanes 0..7 take one 16-token slot each
@@ -785,35 +786,17 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
       }
     } else if (warp == 1) {
-      // ------------------------------------------------------------ MMA issuer
+      // ------------------------------------------------------------ P V issuer
       if (lane == 0) {
-        uint32_t it = 0, n_local = 0;
+        uint32_t it = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
           ItemB bi = decode_b(L, item);
           if (bi.nslot == 0) continue;
           int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
-          if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
-          ++n_local;
-          tc_fence_after();
-          auto qk = [&](uint32_t g, int j) -> bool {
-            int s3 = g % NKB, b = g & 1;
-            if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag)) return false;
-            if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
-            tc_fence_after();
-            issue_qk(tm, sm.q, sm.k[s3], b);
-            mma_commit(&sm.s_full[b]);
-            mma_commit(&sm.k_empty[s3]);
-            if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
-            return true;
-          };
-          ok = qk(it, 0);
           for (int j = 0; j < ntile && ok; ++j) {
             uint32_t g = it + j;
             int s3 = g % NKB, s2 = g % NVB, b = g & 1;
-            // Q K^T of the next tile first, so that it runs while the softmax
-            // works on this one (its K is prefetched three tiles deep)
-            if (j + 1 < ntile && !(ok = qk(g + 1, j + 1))) break;
             if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
                 !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
               ok = false;
@@ -842,8 +825,43 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           it += ntile;
         }
         if (*abort_flag) {
-          mma_commit(&sm.drain);
+          mma_commit(&sm.drain);  // every MMA issued by this thread has completed
           mbar_wait_drain(&sm.drain, 0, kWait);
+        }
+      }
+    } else if (warp == 2) {
+      // ------------------------------------------------------------ Q K^T issuer
+      // A second issuing thread: S = Q K^T of tile g needs only its K copy and
+      // the S/P buffer that P V of tile g - 2 has finished reading.
+      if (lane == 0) {
+        uint32_t it = 0, n_local = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+          ItemB bi = decode_b(L, item);
+          if (bi.nslot == 0) continue;
+          int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
+          if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
+          ++n_local;
+          tc_fence_after();
+          for (int j = 0; j < ntile && ok; ++j) {
+            uint32_t g = it + j;
+            int s3 = g % NKB, b = g & 1;
+            if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag) ||
+                (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_qk(tm, sm.q, sm.k[s3], b);
+            mma_commit(&sm.s_full[b]);
+            mma_commit(&sm.k_empty[s3]);
+            if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
+          }
+          it += ntile;
+        }
+        if (*abort_flag) {
+          mma_commit(&sm.drain2);  // every MMA issued by this thread has completed
+          mbar_wait_drain(&sm.drain2, 0, kWait);
         }
       }
     }
