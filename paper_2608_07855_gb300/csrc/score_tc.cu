@@ -585,7 +585,7 @@ struct SmemB {
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
   uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], meta_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2],
-      s_empty[2], p_full, acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain, drain2;
+      s_empty[2], p_full[2], acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain, drain2;
   uint32_t tmem;
   int abort_flag;
 };
@@ -642,7 +642,11 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       mbar_init(&sm.acc_full[b], 1);
       mbar_init(&sm.acc_empty[b], 4);  // the epilogue warpgroup of that page parity
     }
-    mbar_init(&sm.p_full, 4);
+    // one per S/P buffer: the softmax can finish tile g + 1 before the P V
+    // thread has seen tile g, but not tile g + 2, so a parity wait on a
+    // per-buffer barrier cannot miss a phase
+    mbar_init(&sm.p_full[0], 4);
+    mbar_init(&sm.p_full[1], 4);
     for (int f = 0; f < NFIFO; ++f) {
       mbar_init(&sm.fifo_full[f], 4);
       mbar_init(&sm.fifo_empty[f], 4);
@@ -797,7 +801,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           for (int j = 0; j < ntile && ok; ++j) {
             uint32_t g = it + j;
             int s3 = g % NKB, s2 = g % NVB, b = g & 1;
-            if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
+            if (!mbar_wait(&sm.p_full[b], (g >> 1) & 1, kWait, abort_flag) ||
                 !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
               ok = false;
               break;
@@ -896,8 +900,9 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       for (int j = 0; j < ntile && ok; ++j) {
         uint32_t g = it + j;
         int s = g % NKB, b = g & 1;
-        // the slot table of this stage is published with its K copies
-        if (!mbar_wait(&sm.k_full[s], (g / NKB) & 1, kWait, abort_flag)) {
+        // the slot table of this stage is published with its K copies (warp-
+        // uniform results keep the lanes together for the collective ops)
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.k_full[s], (g / NKB) & 1, kWait, abort_flag))) {
           ok = false;
           break;
         }
@@ -913,7 +918,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
           }
           __syncwarp();
         }
-        if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag))) {
           ok = false;
           break;
         }
@@ -928,6 +933,9 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
 #pragma unroll 1
         for (int ch = 0; ch < BT / 32 && ok; ++ch) {
           float x[32];
+          // tensor-memory loads and stores are warp-collective: the lanes
+          // may have left the bounded waits above on different iterations
+          __syncwarp();
           tmem_ld32f(tm + lane_base + b * BT + 32 * ch, x);
           const SlotMeta m0 = sm.meta[s][2 * ch], m1 = sm.meta[s][2 * ch + 1];
           uint32_t vm = (m0.nv >= SLOT ? 0xffffu : (1u << max(m0.nv, 0)) - 1u) |
@@ -967,8 +975,8 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             n_cur += __popc(h2 ? vm >> 16 : vm & 0xffffu);
             if (mt.flags & 2) {
               int f = po_seen % NFIFO;
-              if (po_seen >= NFIFO &&
-                  !mbar_wait(&sm.fifo_empty[f], ((po_seen / NFIFO) - 1) & 1, kWait, abort_flag)) {
+              if (!__all_sync(0xffffffffu, po_seen < NFIFO || mbar_wait(&sm.fifo_empty[f], ((po_seen / NFIFO) - 1) & 1,
+                                                                           kWait, abort_flag))) {
                 ok = false;
                 break;
               }
@@ -979,11 +987,12 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
             }
           }
         }
+        __syncwarp();
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          mbar_arrive(&sm.p_full);
+          mbar_arrive(&sm.p_full[b]);
           // publish the pages this tile finished to the epilogue
           for (int k = po_first; k < po_seen; ++k) mbar_arrive(&sm.fifo_full[k % NFIFO]);
         }
@@ -1035,8 +1044,8 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       for (int k = 0; k < npages && ok; ++k, ++po) {
         if ((po & 1) != par) continue;
         int f = po % NFIFO;
-        if (!mbar_wait(&sm.fifo_full[f], (po / NFIFO) & 1, kWait, abort_flag) ||
-            !mbar_wait(&sm.acc_full[par], (po >> 1) & 1, kWait, abort_flag)) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.fifo_full[f], (po / NFIFO) & 1, kWait, abort_flag) &&
+                                         mbar_wait(&sm.acc_full[par], (po >> 1) & 1, kWait, abort_flag))) {
           ok = false;
           break;
         }
