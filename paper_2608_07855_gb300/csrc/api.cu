@@ -107,7 +107,7 @@ int cdiv(int a, int b) { return (a + b - 1) / b; }
 int tc_chunk_len(int n_traj, const commitkv_traj *tr) {
   int smax = 0;
   for (int t = 0; t < n_traj; ++t) smax = tr[t].S > smax ? tr[t].S : smax;
-  int c = (smax + 15) / 16;
+  int c = (smax + 7) / 8;  // at most 8 chunks per (layer, KV head)
   if (c < 1024) c = 1024;
   return (c + 127) / 128 * 128;
 }
@@ -162,7 +162,7 @@ size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *
     slots += align_up((size_t)(tr[t].P + 1) * 4) + align_up((size_t)c.nbitem * 32) + kAlign +
              align_up(((size_t)cdiv(tr[t].S, 16) + tr[t].P) * 16);
   }
-  return align_up(items * tc::kRowsPerTile * 132 * 4) + slots;
+  return align_up(items * tc::kPartsPerItem * tc::kRowsPerTile * 132 * 4) + slots;
 }
 
 // Region sizes of each call (bytes after the 256-byte header).
@@ -347,7 +347,7 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
     TcCounts c = tc_counts(shape, trajs[t], CLt);
     items_all += (size_t)shape->layers * shape->kv_heads * tc_chunk_bound(trajs[t].S) * c.nrt;
   }
-  char *slot_base = base + align_up(items_all * tc::kRowsPerTile * 132 * 4);
+  char *slot_base = base + align_up(items_all * tc::kPartsPerItem * tc::kRowsPerTile * 132 * 4);
   for (int b0 = 0; b0 < n_traj; b0 += tc::kMaxTc) {
     int nb = n_traj - b0 < tc::kMaxTc ? n_traj - b0 : tc::kMaxTc;
     memset(&T, 0, sizeof T);

@@ -74,16 +74,20 @@ __device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int ks) {
 }
 
 // ============================================================== pass A
-// TMEM columns: S/P buffers at 0 and 128 (after the softmax reads a 32-column
+// Two softmax warpgroups take alternate tiles of a chunk (global tile g goes
+// to warpgroup g & 1), each with its own S/P buffer, running max, sum and
+// output accumulator, so one warpgroup's softmax overlaps the other's MMAs.
+// TMEM columns: S/P buffer b at 128 b (after the softmax reads a 32-column
 // chunk of S it overwrites the same columns with 16 columns of P_hi and 16
-// of P_lo), O at 256.
+// of P_lo), O_b at 256 + 128 b.  Each item writes two partials, one per
+// warpgroup.
 struct SmemA {
   alignas(1024) uint8_t q[kTileBytes];
   alignas(1024) uint8_t k[NKB][kTileBytes];
   alignas(1024) uint8_t v[NVB][kTileBytes];
-  int pos[4][BT];  // per softmax warp: positions of the current tile
-  uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2], s_empty[2], p_full,
-      pv_done, o_full, o_empty, drain;
+  int pos[2][4][BT];  // per softmax warp: positions of the current tile
+  uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2], s_empty[2], p_full[2],
+      pv_done[2], o_full[2], o_empty[2], drain, drain2;
   uint32_t tmem;
   int abort_flag;
 };
@@ -129,7 +133,7 @@ __device__ __forceinline__ void issue_pv_step(uint32_t tm, uint32_t d_col, const
   mma_bf16_ts(tm + d_col, tm + p_col(b, ks, 1), bd, idesc, 1u);
 }
 
-__global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+__global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   extern __shared__ uint8_t smem_raw[];
   SmemA &sm = *reinterpret_cast<SmemA *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -151,12 +155,13 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.s_full[b], 1);
       mbar_init(&sm.s_empty[b], 1);
+      mbar_init(&sm.p_full[b], 4);
+      mbar_init(&sm.pv_done[b], 1);
+      mbar_init(&sm.o_full[b], 1);
+      mbar_init(&sm.o_empty[b], 4);
     }
-    mbar_init(&sm.p_full, 4);
-    mbar_init(&sm.pv_done, 1);
-    mbar_init(&sm.o_full, 1);
-    mbar_init(&sm.o_empty, 4);
     mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain2, 1);
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -168,104 +173,102 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
   tc_fence_after();
   const uint32_t tm = sm.tmem;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      uint64_t pol = policy_evict_normal();
-      uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
-      bool stop = false;
-      for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x, ++n_local) {
-        if (*abort_flag) break;
-        ItemA a = decode_a(L, item);
-        const TcTraj &tr = L.t[a.t];
-        const TcMaps &mp = L.maps[a.t];
-        if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) break;
-        mbar_expect_tx(&sm.q_full, kTileBytes);
-        int qrow = (a.l * L.Hq + a.kvh * L.g) * tr.W + a.rt * BM;
-        tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
-        tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
-        int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
-        int ntile = (t1 - t0 + BT - 1) / BT;
-        // K of tile g once Q K^T of tile g - 3 is done; V once P V of tile g - 2 is
-        auto load_k = [&](uint32_t g, int tok) -> bool {
-          int s3 = g % NKB;
-          if (g >= NKB && !mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)) return false;
-          mbar_expect_tx(&sm.k_full[s3], kTileBytes);
-          tma4(sm.k[s3], &mp.k, 0, tok, a.kvh, a.l, &sm.k_full[s3], pol);
-          tma4(sm.k[s3] + kHalf, &mp.k, 64, tok, a.kvh, a.l, &sm.k_full[s3], pol);
-          ++n_k;
-          return true;
-        };
-        auto load_v = [&](uint32_t g, int tok) -> bool {
-          int s2 = g % NVB;
-          if (g >= NVB && !mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag)) return false;
-          mbar_expect_tx(&sm.v_full[s2], kTileBytes);
-          tma4(sm.v[s2], &mp.v, 0, tok, a.kvh, a.l, &sm.v_full[s2], pol);
-          tma4(sm.v[s2] + kHalf, &mp.v, 64, tok, a.kvh, a.l, &sm.v_full[s2], pol);
-          ++n_v;
-          return true;
-        };
-        // K runs one tile ahead of V
-        if (ntile > 0) stop = !load_k(it, t0);
-        for (int j = 0; j < ntile && !stop; ++j) {
-          if (j + 1 < ntile && !load_k(it + j + 1, t0 + (j + 1) * BT)) stop = true;
-          else if (!load_v(it + j, t0 + j * BT)) stop = true;
+  // warpgroup 0: TMA producer, P V issuer, Q K^T issuer, one idle warp; 1 and
+  // 2: softmax of the even and the odd tiles.  Register budget per thread:
+  // 56 + 2 x 224 = the launch's 3 x 168.
+  if (warp < 4) {
+    regs_dec<56>();  // warp 3 stays idle
+    if (warp == 0) {
+      // ------------------------------------------------------------ TMA producer
+      if (lane == 0) {
+        uint64_t pol = policy_evict_normal();
+        uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
+        bool stop = false;
+        for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x, ++n_local) {
+          if (*abort_flag) break;
+          ItemA a = decode_a(L, item);
+          const TcTraj &tr = L.t[a.t];
+          const TcMaps &mp = L.maps[a.t];
+          if (n_local > 0 && !mbar_wait(&sm.q_empty, (n_local - 1) & 1, kWait, abort_flag)) break;
+          mbar_expect_tx(&sm.q_full, kTileBytes);
+          int qrow = (a.l * L.Hq + a.kvh * L.g) * tr.W + a.rt * BM;
+          tma_load_2d(sm.q, &mp.q, 0, qrow, &sm.q_full, pol);
+          tma_load_2d(sm.q + kHalf, &mp.q, 64, qrow, &sm.q_full, pol);
+          int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
+          int ntile = (t1 - t0 + BT - 1) / BT;
+          // K of tile g once Q K^T of tile g - 3 is done; V once P V of tile g - 2 is
+          auto load_k = [&](uint32_t g, int tok) -> bool {
+            int s3 = g % NKB;
+            if (g >= NKB && !mbar_wait(&sm.k_empty[s3], ((g / NKB) - 1) & 1, kWait, abort_flag)) return false;
+            mbar_expect_tx(&sm.k_full[s3], kTileBytes);
+            tma4(sm.k[s3], &mp.k, 0, tok, a.kvh, a.l, &sm.k_full[s3], pol);
+            tma4(sm.k[s3] + kHalf, &mp.k, 64, tok, a.kvh, a.l, &sm.k_full[s3], pol);
+            ++n_k;
+            return true;
+          };
+          auto load_v = [&](uint32_t g, int tok) -> bool {
+            int s2 = g % NVB;
+            if (g >= NVB && !mbar_wait(&sm.v_empty[s2], ((g / NVB) - 1) & 1, kWait, abort_flag)) return false;
+            mbar_expect_tx(&sm.v_full[s2], kTileBytes);
+            tma4(sm.v[s2], &mp.v, 0, tok, a.kvh, a.l, &sm.v_full[s2], pol);
+            tma4(sm.v[s2] + kHalf, &mp.v, 64, tok, a.kvh, a.l, &sm.v_full[s2], pol);
+            ++n_v;
+            return true;
+          };
+          // K runs one tile ahead of V
+          if (ntile > 0) stop = !load_k(it, t0);
+          for (int j = 0; j < ntile && !stop; ++j) {
+            if (j + 1 < ntile && !load_k(it + j + 1, t0 + (j + 1) * BT)) stop = true;
+            else if (!load_v(it + j, t0 + j * BT)) stop = true;
+          }
+          it += ntile;
         }
-        it += ntile;
+        if (*abort_flag) {
+          // let the copies already issued land before the CTA leaves
+          for (uint32_t u = (n_k > NKB ? n_k - NKB : 0); u < n_k; ++u)
+            mbar_wait_drain(&sm.k_full[u % NKB], (u / NKB) & 1, kWait);
+          for (uint32_t u = (n_v > NVB ? n_v - NVB : 0); u < n_v; ++u)
+            mbar_wait_drain(&sm.v_full[u % NVB], (u / NVB) & 1, kWait);
+          if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
+        }
       }
-      if (*abort_flag) {
-        // let the copies already issued land before the CTA leaves
-        for (uint32_t u = (n_k > NKB ? n_k - NKB : 0); u < n_k; ++u)
-          mbar_wait_drain(&sm.k_full[u % NKB], (u / NKB) & 1, kWait);
-        for (uint32_t u = (n_v > NVB ? n_v - NVB : 0); u < n_v; ++u)
-          mbar_wait_drain(&sm.v_full[u % NVB], (u / NVB) & 1, kWait);
-        if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
-      }
-    }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+    // ------------------------------------------------------------ P V issuer
     if (lane == 0) {
-      uint32_t it = 0, n_local = 0;
+      uint32_t it = 0;
+      int uses0 = 0, uses1 = 0;  // items in which O_0 / O_1 have been filled so far
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
         ItemA a = decode_a(L, item);
         const TcTraj &tr = L.t[a.t];
         int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
         int ntile = (t1 - t0 + BT - 1) / BT;
-        if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
-        tc_fence_after();
-        auto qk = [&](uint32_t g, int j) -> bool {
-          int s3 = g % NKB, b = g & 1;
-          if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag)) return false;
-          if (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag)) return false;
-          tc_fence_after();
-          issue_qk(tm, sm.q, sm.k[s3], b);
-          mma_commit(&sm.s_full[b]);
-          mma_commit(&sm.k_empty[s3]);
-          if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
-          return true;
-        };
-        if (ntile > 0) ok = qk(it, 0);
-        // the O of the previous item must have been read out before P V overwrites it
-        if (ok && n_local > 0 && !mbar_wait(&sm.o_empty, (n_local - 1) & 1, kWait, abort_flag)) ok = false;
         for (int j = 0; j < ntile && ok; ++j) {
           uint32_t g = it + j;
           int s2 = g % NVB, b = g & 1;
-          // Q K^T of the next tile first, so that it runs while the softmax
-          // works on this one (its K is prefetched three tiles deep)
-          if (j + 1 < ntile && !(ok = qk(g + 1, j + 1))) break;
-          if (!mbar_wait(&sm.p_full, g & 1, kWait, abort_flag) ||
+          const bool first = j < 2, last = j + 2 >= ntile;  // of warpgroup b in this item
+          // O_b of the previous item must have been read out before P V overwrites it
+          const int ub = b ? uses1 : uses0;
+          if (first && ub > 0 && !mbar_wait(&sm.o_empty[b], (ub - 1) & 1, kWait, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait(&sm.p_full[b], (g >> 1) & 1, kWait, abort_flag) ||
               !mbar_wait(&sm.v_full[s2], (g / NVB) & 1, kWait, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
 #pragma unroll
-          for (int ks = 0; ks < BT / 16; ++ks) issue_pv_step(tm, 2 * BT, sm.v[s2], b, ks, j == 0 && ks == 0);
+          for (int ks = 0; ks < BT / 16; ++ks) issue_pv_step(tm, 2 * BT + b * D, sm.v[s2], b, ks, first && ks == 0);
           mma_commit(&sm.s_empty[b]);
           mma_commit(&sm.v_empty[s2]);
-          mma_commit(&sm.pv_done);
-          if (j + 1 == ntile) mma_commit(&sm.o_full);
+          mma_commit(&sm.pv_done[b]);
+          if (last) {
+            mma_commit(&sm.o_full[b]);
+            if (b) ++uses1;
+            else ++uses0;
+          }
         }
         it += ntile;
       }
@@ -274,14 +277,53 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         mbar_wait_drain(&sm.drain, 0, kWait);
       }
     }
+    } else if (warp == 2) {
+      // ------------------------------------------------------------ Q K^T issuer
+      if (lane == 0) {
+        uint32_t it = 0, n_local = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+          ItemA a = decode_a(L, item);
+          const TcTraj &tr = L.t[a.t];
+          int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
+          int ntile = (t1 - t0 + BT - 1) / BT;
+          if (!mbar_wait(&sm.q_full, n_local & 1, kWait, abort_flag)) break;
+          tc_fence_after();
+          for (int j = 0; j < ntile && ok; ++j) {
+            uint32_t g = it + j;
+            int s3 = g % NKB, b = g & 1;
+            if (!mbar_wait(&sm.k_full[s3], (g / NKB) & 1, kWait, abort_flag) ||
+                (g >= 2 && !mbar_wait(&sm.s_empty[b], ((g >> 1) - 1) & 1, kWait, abort_flag))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_qk(tm, sm.q, sm.k[s3], b);
+            mma_commit(&sm.s_full[b]);
+            mma_commit(&sm.k_empty[s3]);
+            if (j + 1 == ntile) mma_commit(&sm.q_empty);  // every Q K^T of this item is issued
+          }
+          it += ntile;
+        }
+        if (*abort_flag) {
+          mma_commit(&sm.drain2);  // every MMA issued by this thread has completed
+          mbar_wait_drain(&sm.drain2, 0, kWait);
+        }
+      }
+    }
   } else {
-    // ------------------------------------------------------------ softmax (warps 2..5)
+    // ------------------------------------------------------------ softmax (warps 4..11)
+    regs_inc<224>();
+    const int hb = (warp - 4) >> 2;   // this warpgroup's tiles: g & 1 == hb
     const int wq = warp & 3;          // TMEM lane quarter of this warp
     const int row = wq * 32 + lane;   // probe row within the tile
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
-    uint32_t it = 0, n_local = 0;
+    const uint32_t o_col = 2 * BT + hb * D;
+    int *posw = sm.pos[hb][wq];
+    uint32_t it = 0;
+    int uses = 0;  // items in which this warpgroup filled O_hb
     bool ok = true;
-    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
       ItemA a = decode_a(L, item);
       const TcTraj &tr = L.t[a.t];
       int rows = L.g * tr.W;
@@ -291,51 +333,53 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
       const int vis_all = tr.prep->vis_all;
       int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
       int ntile = (t1 - t0 + BT - 1) / BT;
+      const int j0 = (hb - (int)it) & 1;  // first tile of this warpgroup in the item
+      float *dst = L.partials + (((int64_t)item * 2 + hb) * BM + row) * (D + 4);
       float m_used = -INFINITY, m_true = -INFINITY, lsum = 0.0f;
       int nvis = 0;
-      for (int j = 0; j < ntile && ok; ++j) {
+      for (int j = j0; j < ntile && ok; j += 2) {
         uint32_t g = it + j;
-        int b = g & 1;
+        const int b = hb;
         int tok0 = t0 + j * BT, nt = min(BT, t1 - tok0);
         // tiles inside the prefix every probe row sees need no position test
         const bool full = tok0 + nt <= vis_all;
         if (!full) {  // each warp keeps its own copy: no cross-warp barrier
           __syncwarp();
 #pragma unroll
-          for (int i = lane; i < BT; i += 32) sm.pos[wq][i] = i < nt ? tr.pos[tok0 + i] : 0x7fffffff;
+          for (int i = lane; i < BT; i += 32) posw[i] = i < nt ? tr.pos[tok0 + i] : 0x7fffffff;
           __syncwarp();
         }
-        if (!mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag)) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full[b], (g >> 1) & 1, kWait, abort_flag))) {
           ok = false;
           break;
         }
         tc_fence_after();
-        float x[BT];
-        tmem_ld32f(tm + lane_base + b * BT + 0, x);
-        tmem_ld32f(tm + lane_base + b * BT + 32, x + 32);
-        tmem_ld32f(tm + lane_base + b * BT + 64, x + 64);
-        tmem_ld32f(tm + lane_base + b * BT + 96, x + 96);
-        tmem_wait_ld();
-        // raw scores: masked ones become -inf; max on the raw scale (scale > 0)
-        int cnt;
-        if (!(full && nt == BT && valid_row)) {
-          cnt = 0;
-#pragma unroll
-          for (int i = 0; i < BT; ++i) {
-            bool vis = valid_row && i < nt && (full || sm.pos[wq][i] <= qp);
-            x[i] = vis ? x[i] : -INFINITY;
-            cnt += vis;
-          }
-        } else {
-          cnt = BT;
-        }
+        // visibility of column i: inside the tile and, outside the prefix every
+        // probe row sees, at or before the row's query position
+        const bool simple = full && nt == BT && valid_row;
+        // sweep 1: row max over the tile, 32 columns at a time
         float mx[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = x[k];
+        for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
+        int cnt = simple ? BT : 0;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BT; c0 += 32) {
+          float x[32];
+          tmem_ld32f(tm + lane_base + b * BT + c0, x);
+          tmem_wait_ld();
+          if (!simple) {
 #pragma unroll
-        for (int i = 8; i < BT; i += 8)
+            for (int i = 0; i < 32; ++i) {
+              bool vis = valid_row && c0 + i < nt && (full || posw[c0 + i] <= qp);
+              x[i] = vis ? x[i] : -INFINITY;
+              cnt += vis;
+            }
+          }
 #pragma unroll
-          for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], x[i + k]);
+          for (int i = 0; i < 32; i += 8)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], x[i + k]);
+        }
         float smax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
         float mt = smax == -INFINITY ? smax : smax * L.scale_log2;
         nvis += cnt;
@@ -344,75 +388,92 @@ __global__ void __launch_bounds__(192, 1) pass_a_tc(const __grid_constant__ TcLa
         bool rescale = m_new > m_used + kLazy;  // false while both are -inf
         float alpha = (rescale && m_used != -INFINITY) ? exp2f(m_used - m_new) : 0.0f;
         if (rescale) m_used = m_new;
-        // P V of the previous tile done: O is stable (phase g-1 of pv_done)
-        if (g > 0 && !mbar_wait(&sm.pv_done, (g - 1) & 1, kWait, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        if (j > 0 && __any_sync(0xffffffffu, rescale)) {
-          float f = rescale ? alpha : 1.0f;
-#pragma unroll
-          for (int c0 = 0; c0 < D; c0 += 32) {
-            uint32_t r[32];
-            tmem_ld32(tm + lane_base + 2 * BT + c0, r);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * f);
-            tmem_st32(tm + lane_base + 2 * BT + c0, r);
+        if (j > j0) {
+          // P V of this warpgroup's previous tile done: O_hb is stable
+          if (!__all_sync(0xffffffffu, mbar_wait(&sm.pv_done[b], ((g >> 1) - 1) & 1, kWait, abort_flag))) {
+            ok = false;
+            break;
           }
-          tmem_wait_st();
+          tc_fence_after();
+          if (__any_sync(0xffffffffu, rescale)) {
+            float f = rescale ? alpha : 1.0f;
+#pragma unroll
+            for (int c0 = 0; c0 < D; c0 += 32) {
+              uint32_t r[32];
+              tmem_ld32(tm + lane_base + o_col + c0, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * f);
+              tmem_st32(tm + lane_base + o_col + c0, r);
+            }
+            tmem_wait_st();
+          }
         }
         if (rescale) lsum *= alpha;
         const float neg_m = m_used == -INFINITY ? 0.0f : -m_used;
-#pragma unroll
-        for (int i = 0; i < BT; ++i) x[i] = fast_exp2(fmaf(x[i], L.scale_log2, neg_m));  // 2^-inf = 0
+        // sweep 2: p = 2^(s c - m) on the visible columns (2^-inf = 0), the row
+        // sum, and P as the (hi, lo) bf16 pair over the S columns just read
         float pacc[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) pacc[k] = x[k];
-#pragma unroll
-        for (int i = 8; i < BT; i += 8)
-#pragma unroll
-          for (int k = 0; k < 8; ++k) pacc[k] += x[i + k];
-        float ps = ((pacc[0] + pacc[1]) + (pacc[2] + pacc[3])) + ((pacc[4] + pacc[5]) + (pacc[6] + pacc[7]));
-#pragma unroll
+        for (int k = 0; k < 8; ++k) pacc[k] = 0.0f;
+#pragma unroll 1
         for (int c0 = 0; c0 < BT; c0 += 32) {
+          float x[32];
+          tmem_ld32f(tm + lane_base + b * BT + c0, x);
+          tmem_wait_ld();
+          if (!simple) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              bool vis = valid_row && c0 + i < nt && (full || posw[c0 + i] <= qp);
+              x[i] = vis ? x[i] : -INFINITY;
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) x[i] = fast_exp2(fmaf(x[i], L.scale_log2, neg_m));
+#pragma unroll
+          for (int i = 0; i < 32; i += 8)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) pacc[k] += x[i + k];
           uint32_t pk[32];
-          split_pack32(x + c0, pk);
+          split_pack32(x, pk);
           tmem_st32(tm + lane_base + b * BT + c0, pk);
         }
+        float ps = ((pacc[0] + pacc[1]) + (pacc[2] + pacc[3])) + ((pacc[4] + pacc[5]) + (pacc[6] + pacc[7]));
         tmem_wait_st();
         lsum += ps;
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_full);
+        if (lane == 0) mbar_arrive(&sm.p_full[b]);
       }
       if (!ok) break;
-      // item done: O complete after the last P V
-      if (!mbar_wait(&sm.o_full, n_local & 1, kWait, abort_flag)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float *dst = L.partials + ((int64_t)item * BM + row) * (D + 4);
-#pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld32(tm + lane_base + 2 * BT + c0, r);
-        tmem_wait_ld();
-        if (valid_row) {
-#pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4 *>(dst + 4 + c0 + i) =
-                make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]), __uint_as_float(r[i + 2]),
-                            __uint_as_float(r[i + 3]));
+      if (j0 < ntile) {
+        // this warpgroup's O is complete after its last P V of the item
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.o_full[hb], uses & 1, kWait, abort_flag))) {
+          ok = false;
+          break;
         }
+        tc_fence_after();
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32(tm + lane_base + o_col + c0, r);
+          tmem_wait_ld();
+          if (valid_row) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              *reinterpret_cast<float4 *>(dst + 4 + c0 + i) =
+                  make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]), __uint_as_float(r[i + 2]),
+                              __uint_as_float(r[i + 3]));
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.o_empty[hb]);
+        ++uses;
       }
-      // (reference max of l and O, sum, visible count, true max)
+      // (reference max of l and O, sum, visible count, true max); a warpgroup
+      // without tiles in this item leaves an empty partial
       if (valid_row) *reinterpret_cast<float4 *>(dst) = make_float4(m_used, lsum, (float)nvis, m_true);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.o_empty);
       it += ntile;
     }
   }
@@ -437,16 +498,18 @@ __global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaun
   int kvh = local % L.H, li = local / L.H;
   int l = L.layer_ids[li];
   int rt = row / BM, rl = row % BM;
-  auto part = [&](int c) {
-    int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + c) * tr.nrt + rt;
-    return L.partials + ((int64_t)item * BM + rl) * (D + 4);
+  // partial k = 2 c + h: chunk c, softmax warpgroup h
+  auto part = [&](int k) {
+    int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + (k >> 1)) * tr.nrt + rt;
+    return L.partials + (((int64_t)item * 2 + (k & 1)) * BM + rl) * (D + 4);
   };
-  float m = -INFINITY;  // true row max over the chunks (base 2)
-  for (int c = 0; c < tr.nchunk; ++c) m = fmaxf(m, part(c)[3]);
+  const int nparts = 2 * tr.nchunk;
+  float m = -INFINITY;  // true row max over the partials (base 2)
+  for (int k = 0; k < nparts; ++k) m = fmaxf(m, part(k)[3]);
   float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
   float lsum = 0.0f, n = 0.0f;
-  for (int c = 0; c < tr.nchunk; ++c) {
-    const float *p = part(c);
+  for (int k = 0; k < nparts; ++k) {
+    const float *p = part(k);
     n += p[2];
     if (p[0] == -INFINITY) continue;
     float a = exp2f(p[0] - m);
@@ -1154,7 +1217,7 @@ cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, in
   if (e != cudaSuccess) return e;
   prep_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
   int na = L.item_off_a[L.n_traj];
-  if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 192, smem_a(), s>>>(L, hdr);
+  if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 384, smem_a(), s>>>(L, hdr);
   int rows = L.row_off[L.n_traj];
   if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
   int nb = L.item_off_b[L.n_traj];

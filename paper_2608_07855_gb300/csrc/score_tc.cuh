@@ -11,6 +11,7 @@ namespace tc {
 constexpr int kMaxTc = 16;          // trajectories per launch (tensor maps travel as parameters)
 constexpr int kRowsPerTile = 128;   // probe rows per MMA tile
 constexpr int kSlotsPerItem = 128;  // 16-token slots per pass-B work item
+constexpr int kPartsPerItem = 2;    // pass-A partials per work item
 
 struct TcMaps {
   CUtensorMap q;             // Q as [M*Hq*W rows][128], box 64 x 128
@@ -41,7 +42,7 @@ struct TcLaunch {
   TcTraj t[kMaxTc];
   int n_traj, M, H, Hq, g, n_layers, chunk_len, slots_per_item;
   float scale_log2;
-  float *partials;  // [items_a][128][132]
+  float *partials;  // [items_a][2][128][132]: one partial per softmax warpgroup
   int item_off_a[kMaxTc + 1], item_off_b[kMaxTc + 1], row_off[kMaxTc + 1];
   uint8_t layer_ids[kMaxLayers];
 };
