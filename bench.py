@@ -197,7 +197,7 @@ def run_ours(args, rank, world, local):
     if st != ck.COMMITKV_OK:
         raise RuntimeError(f"device status after warm-up: {ck.status_string(st)}")
 
-    stage_names = ["score_pre", "score_post", "classify", "joint", "compact"]
+    stage_names = ["score", "classify", "joint", "compact"]
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stage_names) + 1)]
           for _ in range(args.steps)]
     clocks = Clocks(local)
@@ -211,16 +211,14 @@ def run_ours(args, rank, world, local):
     for k in range(args.steps):
         e = ev[k]
         e[0].record(stream)
-        buf.score_pre()
+        buf.score()
         e[1].record(stream)
-        buf.score_post()
-        e[2].record(stream)
         buf.classify()
-        e[3].record(stream)
+        e[2].record(stream)
         buf.joint()
-        e[4].record(stream)
+        e[3].record(stream)
         buf.compact()
-        e[5].record(stream)
+        e[4].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -240,7 +238,7 @@ def run_ours(args, rank, world, local):
     # roofline of the scoring pass (the dominant stage)
     peaks, peak_kind = load_peaks()
     bpt, fpt = algorithmic(cfg)
-    score_ms = stage_ms["score_pre"] + stage_ms["score_post"]
+    score_ms = stage_ms["score"]
     alg_bytes = bpt * tokens_per_step
     alg_flops = fpt * tokens_per_step
     t_mem = alg_bytes / (peaks["hbm_gbs"] * 1e9)
@@ -287,15 +285,16 @@ def run_ours(args, rank, world, local):
 
 def buf_launches(buf):
     """Kernels of this library launched per step (counted from the launch
-    sequence of each call).  Scoring per cache: on the tensor-core path (bf16,
-    head_dim 128) prep + pass A + combine + pass B for every group of up to
-    16 trajectories, else pass A + combine + pass B; classify 1; joint test 1;
-    compaction = select + gather."""
+    sequence of each call).  Scoring, one call over the 2n pre- and
+    post-commit caches: on the tensor-core path (bf16, head_dim 128) prep +
+    pass A + combine + pass B for every group of up to 16 caches, else pass A
+    + combine + pass B; classify 1; joint test 1; compaction = select +
+    gather."""
     cfg = buf.cfg
     tc = cfg.dtype == "bf16" and cfg.d == 128 and os.environ.get("COMMITKV_SCORING") != "simt"
-    n = len(buf.trajs)
+    n = 2 * len(buf.trajs)
     score = 4 * ((n + 15) // 16) if tc else 3
-    return 2 * score + 1 + 1 + 2
+    return score + 1 + 1 + 2
 
 
 def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):

@@ -108,7 +108,9 @@ class StepBuffers:
         self.k_out = [torch.empty(cfg.M, cfg.H, cfg.B, cfg.d, dtype=dt, device=device) for t in trajs]
         self.v_out = [torch.empty(cfg.M, cfg.H, cfg.B, cfg.d, dtype=dt, device=device) for t in trajs]
         self.pos_out = [torch.empty(max(cfg.B, 1), dtype=i32, device=device) for t in trajs]
-        self.ws = ck.alloc_workspace(self.shape, [t.post() for t in trajs], device=device)
+        # sized for the pre- and post-commit caches scored in one call
+        self.ws = ck.alloc_workspace(self.shape, [t.pre() for t in trajs] + [t.post() for t in trajs],
+                                     device=device)
 
     # the five calls ---------------------------------------------------------
     def score_pre(self, stream=None):
@@ -119,6 +121,15 @@ class StepBuffers:
     def score_post(self, stream=None):
         ck.commitkv_page_effects(self.shape, [t.post() for t in self.trajs], self.R_post,
                                  stats_out=self.stats, workspace=self.ws, stream=stream)
+
+    def score(self, stream=None):
+        """R- and R+ (and the post-commit stats) in one call: the pre- and
+        post-commit caches of every trajectory form one batch, so the scoring
+        kernels run once over both."""
+        n = len(self.trajs)
+        ck.commitkv_page_effects(self.shape, [t.pre() for t in self.trajs] + [t.post() for t in self.trajs],
+                                 [r[:t.P_pre] for r, t in zip(self.R_pre, self.trajs)] + self.R_post,
+                                 stats_out=[None] * n + self.stats, workspace=self.ws, stream=stream)
 
     def classify(self, stream=None):
         ck.commitkv_classify([t.P_post for t in self.trajs], self.R_pre, self.R_post,
@@ -138,8 +149,7 @@ class StepBuffers:
                             self.pos_out, workspace=self.ws, stream=stream)
 
     def step(self, stream=None):
-        self.score_pre(stream)
-        self.score_post(stream)
+        self.score(stream)
         self.classify(stream)
         self.joint(stream)
         self.compact(stream)

@@ -279,6 +279,35 @@ def test_batched_trajectories_match_single():
         _assert_close(_np(Rp), o.R_post, 2e-2, "batched R+")
 
 
+def test_pre_and_post_in_one_call():
+    """The pre- and post-commit caches of three trajectories scored in one
+    call (six caches in one launch sequence): effects match the oracle and
+    the separate calls, the post-commit stats match the separate call."""
+    cfgs = [synth.small_config("b0", L_pre=300, L_obs=40), synth.small_config("b1", L_pre=700, L_obs=90),
+            synth.small_config("b2", L_pre=450, L_obs=64)]
+    trs = [synth.make_trajectory(c, 20 + i, traj=i) for i, c in enumerate(cfgs)]
+    devs = [DeviceTrajectory.upload(t) for t in trs]
+    buf = StepBuffers(cfgs[1], devs)
+    buf.score()
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+    one = ([_np(r).copy() for r in buf.R_pre], [_np(r).copy() for r in buf.R_post],
+           [_np(s).copy() for s in buf.stats])
+    buf.score_pre()
+    buf.score_post()
+    torch.cuda.synchronize()
+    assert buf.status() == ck.COMMITKV_OK
+    for i, (t, d) in enumerate(zip(trs, devs)):
+        o = OracleStep(t, "explicit")
+        _assert_close(one[0][i][:d.P_pre], o.R_pre[:d.P_pre], 2e-2, "one-call R-")
+        _assert_close(one[1][i], o.R_post, 2e-2, "one-call R+")
+        _assert_close(one[0][i][:d.P_pre], _np(buf.R_pre[i])[:d.P_pre], 1e-3, "one-call R- vs separate")
+        _assert_close(one[1][i], _np(buf.R_post[i]), 1e-3, "one-call R+ vs separate")
+        a, b = one[2][i].reshape(-1, t.cfg.d + 4), _np(buf.stats[i]).reshape(-1, t.cfg.d + 4)
+        assert np.array_equal(a[:, 2], b[:, 2])
+        _assert_close(a[:, 1], b[:, 1], 1e-5, "one-call row sum vs separate")
+
+
 def test_edge_cases():
     """Empty page list, zero-length pages, a probe row that sees nothing, a
     cache shorter than one tile."""
