@@ -11,7 +11,6 @@
 namespace ckv {
 int simt_rows_per_block();
 int simt_pages_per_block();
-int joint_rows_per_group();
 int compact_max_pending();
 }  // namespace ckv
 
@@ -185,13 +184,11 @@ size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
 }
 
 size_t joint_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, int n_layers) {
-  int g = s->q_heads / s->kv_heads, d = s->head_dim;
-  size_t rows = 0, steps = 0;
-  for (int t = 0; t < n_traj; ++t) {
-    rows += (size_t)n_layers * s->kv_heads * g * tr[t].W;
-    steps += align_up((size_t)tr[t].P * 4);
-  }
-  return 2 * align_up(rows * d * 4) + align_up(rows * 16) + steps;
+  int g = s->q_heads / s->kv_heads, d = s->head_dim, k = joint_round();
+  size_t rows = 0;
+  for (int t = 0; t < n_traj; ++t) rows += (size_t)n_layers * s->kv_heads * g * tr[t].W;
+  return align_up(rows * d * 4) + align_up((size_t)k * rows * d * 4) + align_up(rows * 8) +
+         align_up((size_t)k * rows * 8) + align_up((size_t)3 * n_traj * joint_combos() * 4);
 }
 
 size_t classify_bytes(int n_traj, const int32_t *P) {
@@ -474,28 +471,29 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
   }
   size_t rows_full = 0;
   for (int t = 0; t < n_traj; ++t) rows_full += (size_t)shape->layers * shape->kv_heads * g * post[t].W;
+  const size_t K = (size_t)joint_round(), tab_bytes = (size_t)3 * n_traj * joint_combos() * 4;
   char *base = static_cast<char *>(workspace) + kAlign;
   L.DA = reinterpret_cast<float *>(base);
   base += align_up(rows_full * d * 4);
   L.DE = reinterpret_cast<float *>(base);
-  base += align_up(rows_full * d * 4);
+  base += align_up(K * rows_full * d * 4);
   L.SA = reinterpret_cast<float *>(base);
-  base += align_up(rows_full * 16);
-  char *step_base = base;
+  base += align_up(rows_full * 8);
+  L.SE = reinterpret_cast<float *>(base);
+  base += align_up(K * rows_full * 8);
+  L.roundR = reinterpret_cast<float *>(base);
+  L.rows_full = (int64_t)rows_full;
   for (int t = 0; t < n_traj; ++t) {
     L.stats[t] = stats[t];
     L.cand[t] = cand[t];
     L.accepted[t] = accepted_out[t];
     L.stepR_out[t] = step_R_out ? step_R_out[t] : nullptr;
-    L.stepR[t] = reinterpret_cast<float *>(base);
-    base += align_up((size_t)post[t].P * 4);
   }
   L.n_cand = n_cand;
   L.tau = tau_joint;
-  L.max_steps = maxP;
   cudaError_t e = cudaMemsetAsync(L.DA, 0, rows_total * d * 4, stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(L.SA, 0, rows_full * 16, stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(step_base, 0, (size_t)(base - step_base), stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L.SA, 0, rows_full * 8, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L.roundR, 0, tab_bytes, stream);
   for (int t = 0; t < n_traj && e == cudaSuccess; ++t)
     if (post[t].P > 0) e = cudaMemsetAsync(accepted_out[t], 0, post[t].P, stream);
   // the barrier counters start from a known state

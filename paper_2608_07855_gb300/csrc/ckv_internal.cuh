@@ -139,15 +139,19 @@ struct JointLaunch {
   const int32_t *n_cand;
   uint8_t *accepted[kMaxTraj];
   float *stepR_out[kMaxTraj];
-  float *stepR[kMaxTraj];   // workspace [P_t]
-  float *DA;                // workspace [total rows][d]
-  float *DE;                // workspace [total rows][d]
-  float *SA;                // workspace [total rows] x 4: S_A, n_A, S_E, n_E
+  float *DA;                // workspace [rows_full][d]: D_A of every row
+  float *DE;                // workspace [round][rows_full][d]: D_c of the round's candidates
+  float *SA;                // workspace [rows_full][2]: S_A, n_A
+  float *SE;                // workspace [round][rows_full][2]: S_c, n_c
+  float *roundR;            // workspace [3][n_traj][combos]: per-round tables of row maxima
+  int64_t rows_full;        // rows of all layers, the stride of DE and SE
   int32_t row_off[kMaxTraj + 1];
   float tau;
-  int32_t max_steps;        // upper bound on n_cand (max P_t)
 };
 cudaError_t launch_joint(const JointLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count);
+int joint_rows_per_group();
+int joint_round();   // candidates per round
+int joint_combos();  // (candidate, earlier subset) pairs per round
 
 struct CompactLaunch {
   int32_t n_traj, M, H, d, elem_bytes;

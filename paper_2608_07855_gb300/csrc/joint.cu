@@ -1,17 +1,26 @@
 // Greedy joint test (Section 3.4, Eq. 11; inner loop of Algorithm 1).
 //
-// One cooperative persistent kernel.  Every block owns fixed groups of 64
-// probe rows (trajectory, selected layer, KV head, row block).  Step j:
-//   phase 1  each row computes, for the candidate page E = cand[j],
-//            S_E = sum e_i, U_E = sum e_i v_i (e_i = exp(s_i - m), final m
-//            of the post-commit pass) and D_E = U_E - S_E o; with the sums of
-//            the accepted set A it evaluates
-//            r = ||D_A + D_E|| / ((l - S_A - S_E) ||o||)   (Eq. 6 on A u {E})
-//            and max-reduces r into stepR[j] (Eq. 7);
+// One cooperative persistent kernel.  Every block owns fixed groups of 16
+// probe rows (trajectory, selected layer, KV head, row block).  The
+// candidates are taken in rounds of kRound:
+//   phase 1  each row loads its accepted-set sums (D_A = sum over A of
+//            U_E - S_E o, S_A, n_A) once, then computes for every candidate E
+//            of the round S_E = sum e_i, n_E and D_E = U_E - S_E o (e_i =
+//            exp(s_i - m) with the final m of the post-commit pass).  For each
+//            candidate c and each subset B of the round's earlier candidates
+//            it evaluates Eq. 6 on A u B u {E_c},
+//              r = ||D_A + D_B + D_c|| / ((l - S_A - S_B - S_c) ||o||),
+//            adding the sums in candidate order, which is the order in which
+//            the one-candidate-at-a-time scan would have added them; the max
+//            over rows of each (c, B) goes to a per-round table (Eq. 7);
 //   barrier  (bounded wait: a timeout sets COMMITKV_ERR_TIMEOUT and ends);
-//   phase 2  every row reads stepR[j]; if it is <= tau the row adds D_E,
-//            S_E, n_E into its accepted sums.  Deletion sums over disjoint
-//            pages add, which is what Eq. 11's joint deletion needs.
+//   phase 2  every block replays the round's decisions from the table:
+//            candidate c is accepted iff its value for B = the round's
+//            candidates accepted before it is <= tau, then adds the accepted
+//            D_c, S_c, n_c into its rows' sums, in candidate order.
+// The decisions and step values are those of the scan that takes one
+// candidate per barrier; deletion sums over disjoint pages add, which is what
+// Eq. 11's joint deletion needs.
 #include <cooperative_groups.h>
 
 #include "ckv_internal.cuh"
@@ -22,11 +31,18 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kRB = 64;
-constexpr int kRowsPerWarp = kRB / kWarps;
-constexpr int kTK = 64;
+constexpr int kRowsPerWarp = 2;
+constexpr int kRB = kWarps * kRowsPerWarp;  // rows per group
+constexpr int kTK = 64;                     // page tokens per shared-memory chunk
+constexpr int kRound = 4;                   // candidates per round
+constexpr int kCombos = (1 << kRound) - 1;  // (candidate, subset of the earlier ones) pairs
 constexpr float kNegInf = -__builtin_huge_valf();
 constexpr uint64_t kWaitNs = 1000000000ull;  // 1 s per barrier
+
+static_assert(kRound * 4 <= 32, "accepted masks travel in one word");
+
+// Table slot of candidate c with the subset s of candidates 0..c-1.
+__host__ __device__ constexpr int combo(int c, int s) { return (1 << c) - 1 + s; }
 
 __device__ __forceinline__ int find_group_traj(const int32_t *off, int n, int unit) {
   int t = 0;
@@ -73,211 +89,358 @@ __device__ bool grid_barrier(WsHeader *hdr, unsigned nblocks) {
   return s_ok != 0;
 }
 
-template <typename T, int D>
-__device__ void load_group(const JointLaunch &L, const TrajDev &tr, int l, int kvh, int row0,
-                           int rows, float *sQ) {
-  const Batch &b = L.batch;
-  const T *q = static_cast<const T *>(tr.q);
-  for (int e = threadIdx.x; e < kRB * D; e += kThreads) {
-    int r = e / D, c = e % D, row = row0 + r;
-    float v = 0.0f;
-    if (row < rows) {
-      int h = kvh * b.g + row / tr.W, w = row % tr.W;
-      v = to_f32(q[(((int64_t)l * b.Hq + h) * tr.W + w) * D + c]);
-    }
-    sQ[r * D + c] = v;
+// J consecutive floats (J = 2 or 4) as one vector access.
+template <int J>
+__device__ __forceinline__ void lds_vec(const float *p, float (&v)[J]) {
+  if constexpr (J == 4) {
+    float4 x = *reinterpret_cast<const float4 *>(p);
+    v[0] = x.x, v[1] = x.y, v[2] = x.z, v[3] = x.w;
+  } else {
+    float2 x = *reinterpret_cast<const float2 *>(p);
+    v[0] = x.x, v[1] = x.y;
+  }
+}
+template <int J>
+__device__ __forceinline__ void sts_vec(float *p, const float (&v)[J]) {
+  if constexpr (J == 4) *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  else *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+}
+// 16 bytes of K or V (8 bf16 or 4 floats) as floats: one vector load when the
+// address allows it, else element loads.
+template <typename T>
+__device__ __forceinline__ void load16_f32(const T *p, float (&out)[16 / sizeof(T)]) {
+  constexpr int n = 16 / sizeof(T);
+  if ((reinterpret_cast<uintptr_t>(p) & 15) == 0) {
+    const uint4 raw = *reinterpret_cast<const uint4 *>(p);
+    const T *e = reinterpret_cast<const T *>(&raw);
+#pragma unroll
+    for (int u = 0; u < n; ++u) out[u] = to_f32(e[u]);
+  } else {
+#pragma unroll
+    for (int u = 0; u < n; ++u) out[u] = to_f32(p[u]);
   }
 }
 
+struct Group {
+  int t, l, li, kvh, rows, row0;
+};
+
+__device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
+  const Batch &b = L.batch;
+  Group G;
+  G.t = find_group_traj(L.group_off, b.n_traj, grp);
+  int local = grp - L.group_off[G.t], nrb = L.nrb[G.t];
+  int rb = local % nrb;
+  local /= nrb;
+  G.kvh = local % b.H;
+  G.li = local / b.H;
+  G.l = b.layer_ids[G.li];
+  G.rows = b.g * b.t[G.t].W;
+  G.row0 = rb * kRB;
+  return G;
+}
+
+// Candidates of round r for trajectory t (0 when the scan is over).
+__device__ __forceinline__ int round_count(const JointLaunch &L, int t, int r) {
+  int nc = min(max(L.n_cand[t], 0), L.batch.t[t].P);
+  return max(0, min(kRound, nc - r * kRound));
+}
+
+// The round's decisions, replayed from its table: bit c set = accepted.
+__device__ __forceinline__ unsigned resolve_round(const float *tab, int kc, float tau) {
+  unsigned acc = 0;
+  for (int c = 0; c < kc; ++c) {
+    float R = *(volatile const float *)(tab + combo(c, acc));
+    if (R <= tau) acc |= 1u << c;
+  }
+  return acc;
+}
+
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads) joint_kernel(const __grid_constant__ JointLaunch L,
+__global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constant__ JointLaunch L,
                                                          WsHeader *hdr) {
   extern __shared__ float smem[];
-  float *sQ = smem;
-  float *sK = sQ + kRB * D;
-  float *sV = sK + kTK * (D + 1);
+  float *sQ = smem;                           // [kRB][D]
+  float *sK = sQ + kRB * D;                   // [kTK][D + 4]
+  float *sV = sK + kTK * (D + 4);             // [kTK][D]
   int *sPos = reinterpret_cast<int *>(sV + kTK * D);
-  float *sP = reinterpret_cast<float *>(sPos + kTK);
-  __shared__ float s_rmax;
+  float *sP = reinterpret_cast<float *>(sPos + kTK);  // [kWarps][kTK][kRowsPerWarp]
+  __shared__ float s_rmax[kCombos];
+  // Each lane owns J = D / 32 consecutive channels (J * lane ..) of every
+  // row, so that V, D_c and D_A move as one vector per lane.
   constexpr int J = D / 32;
   const Batch &b = L.batch;
-  int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  int ngroups = L.group_off[b.n_traj];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int ngroups = L.group_off[b.n_traj];
+  const int64_t rows_full = L.rows_full;
 
-  int steps = 0;
-  for (int t = 0; t < b.n_traj; ++t) steps = max(steps, min(max(L.n_cand[t], 0), b.t[t].P));
+  int rounds = 0;
+  for (int t = 0; t < b.n_traj; ++t) {
+    int nc = min(max(L.n_cand[t], 0), b.t[t].P);
+    rounds = max(rounds, (nc + kRound - 1) / kRound);
+  }
 
-  for (int j = 0; j < steps; ++j) {
-    // ---------------- phase 1: evaluate R+(A u {E_j}) on this block's rows
+  for (int r = 0; r < rounds; ++r) {
+    float *tab_r = L.roundR + (size_t)(r % 3) * b.n_traj * kCombos;
+    // ---------------- phase 1: the round's candidates on this block's rows
     for (int grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
-      int t = find_group_traj(L.group_off, b.n_traj, grp);
-      const TrajDev &tr = b.t[t];
-      int nc = min(max(L.n_cand[t], 0), tr.P);
-      if (j >= nc) continue;
-      int E = L.cand[t][j];
-      if (E < 0 || E >= tr.P) {
-        if (threadIdx.x == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, -4);
-        continue;
-      }
-      int local = grp - L.group_off[t], nrb = L.nrb[t];
-      int rb = local % nrb;
-      local /= nrb;
-      int kvh = local % b.H, li = local / b.H;
-      int l = b.layer_ids[li];
-      int rows = b.g * tr.W, row0 = rb * kRB;
+      const Group G = decode_group(L, grp);
+      const TrajDev &tr = b.t[G.t];
+      const int kc = round_count(L, G.t, r);
+      if (kc == 0) continue;
       __syncthreads();
-      load_group<T, D>(L, tr, l, kvh, row0, rows, sQ);
-      if (threadIdx.x == 0) s_rmax = 0.0f;
+      for (int e = threadIdx.x; e < kRB * D; e += kThreads) {
+        int rr = e / D, c = e % D, row = G.row0 + rr;
+        float v = 0.0f;
+        if (row < G.rows) {
+          int h = G.kvh * b.g + row / tr.W, w = row % tr.W;
+          v = to_f32(static_cast<const T *>(tr.q)[(((int64_t)G.l * b.Hq + h) * tr.W + w) * D + c]);
+        }
+        sQ[rr * D + c] = v;
+      }
+      if (threadIdx.x < kCombos) s_rmax[threadIdx.x] = 0.0f;
       __syncthreads();
 
-      float m2[kRowsPerWarp], lsum[kRowsPerWarp], onorm[kRowsPerWarp], o[kRowsPerWarp][J];
-      float S_E[kRowsPerWarp], U[kRowsPerWarp][J];
-      int nvis[kRowsPerWarp], n_E[kRowsPerWarp], qp[kRowsPerWarp];
+      float m2[kRowsPerWarp], lsum[kRowsPerWarp], onorm[kRowsPerWarp], o[kRowsPerWarp][J], DA[kRowsPerWarp][J];
+      float SA[kRowsPerWarp];
+      int nA[kRowsPerWarp], nvis[kRowsPerWarp], qp[kRowsPerWarp];
       bool okr[kRowsPerWarp];
+      int64_t grow[kRowsPerWarp];
 #pragma unroll
       for (int k = 0; k < kRowsPerWarp; ++k) {
-        int row = row0 + warp * kRowsPerWarp + k;
-        okr[k] = row < rows;
-        int h = kvh * b.g + (okr[k] ? row / tr.W : 0), w = okr[k] ? row % tr.W : 0;
-        const float *st = L.stats[t] + (((int64_t)l * b.Hq + h) * tr.W + w) * (D + 4);
+        int row = G.row0 + warp * kRowsPerWarp + k;
+        okr[k] = row < G.rows;
+        int h = G.kvh * b.g + (okr[k] ? row / tr.W : 0), w = okr[k] ? row % tr.W : 0;
+        grow[k] = L.row_off[G.t] + (int64_t)(G.li * b.H + G.kvh) * G.rows + (okr[k] ? row : 0);
+        const float *st = L.stats[G.t] + (((int64_t)G.l * b.Hq + h) * tr.W + w) * (D + 4);
         float mn = okr[k] ? st[0] : kNegInf;
         m2[k] = mn == kNegInf ? mn : mn * 1.4426950408889634f;
         lsum[k] = okr[k] ? st[1] : 0.0f;
         nvis[k] = okr[k] ? (int)st[2] : 0;
         qp[k] = okr[k] ? tr.qpos[w] : -0x7fffffff;
+        const float *da = L.DA + grow[k] * D;
         float ss = 0.0f;
 #pragma unroll
         for (int jj = 0; jj < J; ++jj) {
-          o[k][jj] = okr[k] ? st[4 + lane + 32 * jj] : 0.0f;
+          const int ch = J * lane + jj;
+          o[k][jj] = okr[k] ? st[4 + ch] : 0.0f;
           ss = fmaf(o[k][jj], o[k][jj], ss);
-          U[k][jj] = 0.0f;
+          DA[k][jj] = okr[k] ? da[ch] : 0.0f;
         }
         onorm[k] = sqrtf(warp_sum(ss));
-        S_E[k] = 0.0f;
-        n_E[k] = 0;
+        SA[k] = okr[k] ? L.SA[grow[k] * 2] : 0.0f;
+        nA[k] = okr[k] ? (int)L.SA[grow[k] * 2 + 1] : 0;
       }
-      int ps = tr.ps[E], pl = tr.pl[E];
-      if (pl < 0 || ps < 0 || ps > tr.S - pl) {
-        if (threadIdx.x == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, E);
-        pl = 0;
-        ps = 0;
-      }
-      const T *kp = static_cast<const T *>(tr.k) + (int64_t)l * tr.sl + (int64_t)kvh * tr.sh;
-      const T *vp = static_cast<const T *>(tr.v) + (int64_t)l * tr.sl + (int64_t)kvh * tr.sh;
-      for (int tok0 = ps; tok0 < ps + pl; tok0 += kTK) {
-        int nt = min(kTK, ps + pl - tok0);
-        __syncthreads();
-        for (int e = threadIdx.x; e < kTK * D; e += kThreads) {
-          int i = e / D, c = e % D;
-          float kv = 0.0f, vv = 0.0f;
-          if (i < nt) {
-            int64_t off = (int64_t)(tok0 + i) * tr.st + c;
-            kv = to_f32(kp[off]);
-            vv = to_f32(vp[off]);
-          }
-          sK[i * (D + 1) + c] = kv;
-          sV[i * D + c] = vv;
-        }
-        for (int i = threadIdx.x; i < kTK; i += kThreads) sPos[i] = i < nt ? tr.pos[tok0 + i] : 0;
-        __syncthreads();
-#pragma unroll 1
+
+      // D_c, S_c, n_c of each candidate of the round
+      float DE[kRound][kRowsPerWarp][J], SE[kRound][kRowsPerWarp];
+      int nE[kRound][kRowsPerWarp];
+#pragma unroll
+      for (int c = 0; c < kRound; ++c) {
+        float U[kRowsPerWarp][J], S_c[kRowsPerWarp];
+        int n_c[kRowsPerWarp];
+#pragma unroll
         for (int k = 0; k < kRowsPerWarp; ++k) {
-          if (!okr[k]) continue;
-          const float *q = sQ + (warp * kRowsPerWarp + k) * D;
-          bool v0 = lane < nt && sPos[lane] <= qp[k], v1 = lane + 32 < nt && sPos[lane + 32] <= qp[k];
-          float s0 = 0.0f, s1 = 0.0f;
-          if (v0)
-            for (int c = 0; c < D; ++c) s0 = fmaf(q[c], sK[lane * (D + 1) + c], s0);
-          if (v1)
-            for (int c = 0; c < D; ++c) s1 = fmaf(q[c], sK[(lane + 32) * (D + 1) + c], s1);
-          float e0 = v0 ? exp2f(s0 * b.scale_log2 - m2[k]) : 0.0f;
-          float e1 = v1 ? exp2f(s1 * b.scale_log2 - m2[k]) : 0.0f;
-          S_E[k] += warp_sum(e0 + e1);
-          n_E[k] += __popc(__ballot_sync(0xffffffffu, v0)) + __popc(__ballot_sync(0xffffffffu, v1));
-          float *pw = sP + warp * kTK;
-          pw[lane] = e0;
-          pw[lane + 32] = e1;
-          __syncwarp();
-          for (int i = 0; i < nt; ++i) {
-            float p = pw[i];
+          S_c[k] = 0.0f;
+          n_c[k] = 0;
 #pragma unroll
-            for (int jj = 0; jj < J; ++jj) U[k][jj] = fmaf(p, sV[i * D + lane + 32 * jj], U[k][jj]);
+          for (int jj = 0; jj < J; ++jj) U[k][jj] = 0.0f;
+        }
+        int ps = 0, pl = 0;
+        if (c < kc) {
+          int E = L.cand[G.t][r * kRound + c];
+          if (E < 0 || E >= tr.P) {
+            if (threadIdx.x == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, -4);
+          } else {
+            ps = tr.ps[E];
+            pl = tr.pl[E];
+            if (pl < 0 || ps < 0 || ps > tr.S - pl) {
+              if (threadIdx.x == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, E);
+              pl = 0;
+              ps = 0;
+            }
+          }
+        }
+        const T *kp = static_cast<const T *>(tr.k) + (int64_t)G.l * tr.sl + (int64_t)G.kvh * tr.sh;
+        const T *vp = static_cast<const T *>(tr.v) + (int64_t)G.l * tr.sl + (int64_t)G.kvh * tr.sh;
+        for (int tok0 = ps; tok0 < ps + pl; tok0 += kTK) {
+          const int nt = min(kTK, ps + pl - tok0);
+          __syncthreads();
+          constexpr int V8 = 16 / sizeof(T);  // elements per 16-byte load
+          for (int e = threadIdx.x; e < kTK * D / V8; e += kThreads) {
+            const int i = e / (D / V8), ch = (e % (D / V8)) * V8;
+            float kv[V8], vv[V8];
+            if (i < nt) {
+              const int64_t off = (int64_t)(tok0 + i) * tr.st + ch;
+              load16_f32<T>(kp + off, kv);
+              load16_f32<T>(vp + off, vv);
+            } else {
+#pragma unroll
+              for (int u = 0; u < V8; ++u) kv[u] = vv[u] = 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < V8; u += 4) {
+              *reinterpret_cast<float4 *>(sK + i * (D + 4) + ch + u) = make_float4(kv[u], kv[u + 1], kv[u + 2], kv[u + 3]);
+              *reinterpret_cast<float4 *>(sV + i * D + ch + u) = make_float4(vv[u], vv[u + 1], vv[u + 2], vv[u + 3]);
+            }
+          }
+          for (int i = threadIdx.x; i < kTK; i += kThreads) sPos[i] = i < nt ? tr.pos[tok0 + i] : 0;
+          __syncthreads();
+          // scores of tokens lane and lane + 32 for the warp's rows (the four
+          // dot products run side by side; each keeps its channel order)
+          const float *q0 = sQ + (warp * kRowsPerWarp) * D;
+          float s[kRowsPerWarp][2];
+#pragma unroll
+          for (int k = 0; k < kRowsPerWarp; ++k) s[k][0] = s[k][1] = 0.0f;
+          const bool in0 = lane < nt, in1 = lane + 32 < nt;
+#pragma unroll 2
+          for (int ch = 0; ch < D; ch += 4) {
+            const float4 k0 = *reinterpret_cast<const float4 *>(sK + lane * (D + 4) + ch);
+            const float4 k1 = *reinterpret_cast<const float4 *>(sK + (lane + 32) * (D + 4) + ch);
+#pragma unroll
+            for (int k = 0; k < kRowsPerWarp; ++k) {
+              const float4 qv = *reinterpret_cast<const float4 *>(q0 + k * D + ch);
+              s[k][0] = fmaf(qv.x, k0.x, s[k][0]);
+              s[k][0] = fmaf(qv.y, k0.y, s[k][0]);
+              s[k][0] = fmaf(qv.z, k0.z, s[k][0]);
+              s[k][0] = fmaf(qv.w, k0.w, s[k][0]);
+              s[k][1] = fmaf(qv.x, k1.x, s[k][1]);
+              s[k][1] = fmaf(qv.y, k1.y, s[k][1]);
+              s[k][1] = fmaf(qv.z, k1.z, s[k][1]);
+              s[k][1] = fmaf(qv.w, k1.w, s[k][1]);
+            }
+          }
+          float *pw = sP + warp * kRowsPerWarp * kTK;  // [token][row]
+#pragma unroll
+          for (int k = 0; k < kRowsPerWarp; ++k) {
+            bool v0 = okr[k] && in0 && sPos[lane] <= qp[k], v1 = okr[k] && in1 && sPos[lane + 32] <= qp[k];
+            float e0 = v0 ? exp2f(s[k][0] * b.scale_log2 - m2[k]) : 0.0f;
+            float e1 = v1 ? exp2f(s[k][1] * b.scale_log2 - m2[k]) : 0.0f;
+            S_c[k] += warp_sum(e0 + e1);
+            n_c[k] += __popc(__ballot_sync(0xffffffffu, v0)) + __popc(__ballot_sync(0xffffffffu, v1));
+            pw[lane * kRowsPerWarp + k] = e0;
+            pw[(lane + 32) * kRowsPerWarp + k] = e1;
+          }
+          __syncwarp();
+          static_assert(kRowsPerWarp == 2, "the weights of a token are read as one float2");
+          for (int i = 0; i < nt; ++i) {
+            const float2 p = *reinterpret_cast<const float2 *>(pw + i * kRowsPerWarp);
+            float v[J];
+            lds_vec<J>(sV + i * D + J * lane, v);
+#pragma unroll
+            for (int jj = 0; jj < J; ++jj) {
+              U[0][jj] = fmaf(p.x, v[jj], U[0][jj]);
+              U[1][jj] = fmaf(p.y, v[jj], U[1][jj]);
+            }
           }
           __syncwarp();
         }
-      }
-      float rmax = 0.0f;
 #pragma unroll
-      for (int k = 0; k < kRowsPerWarp; ++k) {
-        if (!okr[k]) continue;
-        int64_t grow = L.row_off[t] + (int64_t)(li * b.H + kvh) * rows + row0 + warp * kRowsPerWarp + k;
-        float *DA = L.DA + grow * D;
-        float *DE = L.DE + grow * D;
-        float *SA = L.SA + grow * 4;
-        float ss = 0.0f;
+        for (int k = 0; k < kRowsPerWarp; ++k) {
+          SE[c][k] = S_c[k];
+          nE[c][k] = n_c[k];
 #pragma unroll
-        for (int jj = 0; jj < J; ++jj) {
-          float de = fmaf(-S_E[k], o[k][jj], U[k][jj]);
-          DE[lane + 32 * jj] = de;
-          float dsum = DA[lane + 32 * jj] + de;
-          ss = fmaf(dsum, dsum, ss);
-        }
-        float num2 = warp_sum(ss);
-        float S_tot = SA[0] + S_E[k];
-        int n_tot = (int)SA[1] + n_E[k];
-        float r = effect_value(n_tot, nvis[k], S_tot, lsum[k], num2, onorm[k]);
-        rmax = fmaxf(rmax, r);
-        if (lane == 0) {
-          SA[2] = S_E[k];
-          SA[3] = (float)n_E[k];
+          for (int jj = 0; jj < J; ++jj) DE[c][k][jj] = fmaf(-S_c[k], o[k][jj], U[k][jj]);
+          if (c < kc && okr[k]) {
+            sts_vec<J>(L.DE + ((int64_t)c * rows_full + grow[k]) * D + J * lane, DE[c][k]);
+            if (lane == 0) {
+              L.SE[((int64_t)c * rows_full + grow[k]) * 2] = S_c[k];
+              L.SE[((int64_t)c * rows_full + grow[k]) * 2 + 1] = (float)n_c[k];
+            }
+          }
         }
       }
-      if (lane == 0) atomicMax(reinterpret_cast<int *>(&s_rmax), __float_as_int(rmax));
+
+      // Eq. 6 on A u B u {E_c} for every candidate c and subset B of the
+      // earlier ones, sums added in candidate order
+#pragma unroll
+      for (int c = 0; c < kRound; ++c) {
+        if (c >= kc) break;
+#pragma unroll 1
+        for (int sb = 0; sb < (1 << c); ++sb) {
+          float rmax = 0.0f;
+#pragma unroll
+          for (int k = 0; k < kRowsPerWarp; ++k) {
+            float x[J], S_tot = SA[k];
+            int n_tot = nA[k];
+#pragma unroll
+            for (int jj = 0; jj < J; ++jj) x[jj] = DA[k][jj];
+#pragma unroll
+            for (int bb = 0; bb < kRound - 1; ++bb) {
+              if (bb < c && ((sb >> bb) & 1)) {
+#pragma unroll
+                for (int jj = 0; jj < J; ++jj) x[jj] += DE[bb][k][jj];
+                S_tot += SE[bb][k];
+                n_tot += nE[bb][k];
+              }
+            }
+            float ss = 0.0f;
+#pragma unroll
+            for (int jj = 0; jj < J; ++jj) {
+              float dsum = x[jj] + DE[c][k][jj];
+              ss = fmaf(dsum, dsum, ss);
+            }
+            float num2 = warp_sum(ss);
+            float rr = effect_value(n_tot + nE[c][k], nvis[k], S_tot + SE[c][k], lsum[k], num2, onorm[k]);
+            if (okr[k]) rmax = fmaxf(rmax, rr);
+          }
+          if (lane == 0) atomicMax(reinterpret_cast<int *>(&s_rmax[combo(c, sb)]), __float_as_int(rmax));
+        }
+      }
       __syncthreads();
-      if (threadIdx.x == 0) atomic_max_nonneg(L.stepR[t] + j, s_rmax);
+      if (threadIdx.x < kCombos && threadIdx.x < combo(kc, 0))
+        atomic_max_nonneg(tab_r + G.t * kCombos + threadIdx.x, s_rmax[threadIdx.x]);
     }
-    // ---------------- barrier: every block's contribution to stepR[j] is in
+    // ---------------- barrier: every block's part of the round's table is in
     if (!grid_barrier(hdr, gridDim.x)) return;
-    // ---------------- phase 2: accept or reject, add the accepted sums
+    // ---------------- phase 2: replay the decisions, add the accepted sums
     for (int grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
-      int t = find_group_traj(L.group_off, b.n_traj, grp);
-      const TrajDev &tr = b.t[t];
-      int nc = min(max(L.n_cand[t], 0), tr.P);
-      if (j >= nc) continue;
-      int E = L.cand[t][j];
-      if (E < 0 || E >= tr.P) continue;
-      float R = *(volatile float *)(L.stepR[t] + j);
-      if (!(R <= L.tau)) continue;
-      int local = grp - L.group_off[t], nrb = L.nrb[t];
-      int rb = local % nrb;
-      local /= nrb;
-      int kvh = local % b.H, li = local / b.H;
-      int rows = b.g * tr.W, row0 = rb * kRB;
+      const Group G = decode_group(L, grp);
+      const int kc = round_count(L, G.t, r);
+      if (kc == 0) continue;
+      const unsigned acc = resolve_round(tab_r + G.t * kCombos, kc, L.tau);
+      if (acc == 0) continue;
 #pragma unroll 1
       for (int k = 0; k < kRowsPerWarp; ++k) {
-        int row = row0 + warp * kRowsPerWarp + k;
-        if (row >= rows) continue;
-        int64_t grow = L.row_off[t] + (int64_t)(li * b.H + kvh) * rows + row;
-        float *DA = L.DA + grow * D;
-        const float *DE = L.DE + grow * D;
-        float *SA = L.SA + grow * 4;
+        int row = G.row0 + warp * kRowsPerWarp + k;
+        if (row >= G.rows) continue;
+        int64_t gr = L.row_off[G.t] + (int64_t)(G.li * b.H + G.kvh) * G.rows + row;
+        float *da = L.DA + gr * D;
+        float *sa = L.SA + gr * 2;
+        for (int c = 0; c < kc; ++c) {
+          if (!((acc >> c) & 1u)) continue;
+          const float *de = L.DE + ((int64_t)c * rows_full + gr) * D;
 #pragma unroll
-        for (int jj = 0; jj < J; ++jj) DA[lane + 32 * jj] += DE[lane + 32 * jj];
-        if (lane == 0) {
-          SA[0] += SA[2];
-          SA[1] += SA[3];
+          for (int jj = 0; jj < J; ++jj) {
+            const int ch = J * lane + jj;
+            da[ch] += de[ch];
+          }
+          if (lane == 0) {
+            sa[0] += L.SE[((int64_t)c * rows_full + gr) * 2];
+            sa[1] += L.SE[((int64_t)c * rows_full + gr) * 2 + 1];
+          }
         }
       }
     }
     if (blockIdx.x == 0) {
       for (int t = threadIdx.x; t < b.n_traj; t += kThreads) {
-        const TrajDev &tr = b.t[t];
-        int nc = min(max(L.n_cand[t], 0), tr.P);
-        if (j >= nc) continue;
-        int E = L.cand[t][j];
-        float R = *(volatile float *)(L.stepR[t] + j);
-        if (L.stepR_out[t]) L.stepR_out[t][j] = R;
-        if (E >= 0 && E < tr.P && R <= L.tau) L.accepted[t][E] = 1;
+        const int kc = round_count(L, t, r);
+        float *tab = tab_r + t * kCombos;
+        unsigned acc = 0;
+        for (int c = 0; c < kc; ++c) {
+          const int j = r * kRound + c;
+          const int E = L.cand[t][j];
+          const float R = *(volatile float *)(tab + combo(c, acc));
+          if (L.stepR_out[t]) L.stepR_out[t][j] = R;
+          if (R <= L.tau) {
+            acc |= 1u << c;
+            if (E >= 0 && E < b.t[t].P) L.accepted[t][E] = 1;
+          }
+        }
+        // the table of round r + 2 starts from zero (the last reads of this
+        // slot were in phase 2 of round r - 1, before this round's barrier)
+        float *next = L.roundR + (size_t)((r + 2) % 3) * b.n_traj * kCombos + t * kCombos;
+        for (int i = 0; i < kCombos; ++i) next[i] = 0.0f;
       }
     }
   }
@@ -285,7 +448,7 @@ __global__ void __launch_bounds__(kThreads) joint_kernel(const __grid_constant__
 
 template <typename T, int D>
 cudaError_t launch_joint_typed(const JointLaunch &L, WsHeader *hdr, cudaStream_t s, int sm_count) {
-  size_t smem = (size_t)(kRB * D + kTK * (D + 1) + kTK * D) * 4 + kTK * 4 + kWarps * kTK * 4;
+  size_t smem = (size_t)(kRB * D + kTK * (D + 4) + kTK * D) * 4 + kTK * 4 + kWarps * kRowsPerWarp * kTK * 4;
   cudaError_t e = cudaFuncSetAttribute(joint_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
@@ -314,6 +477,8 @@ cudaError_t launch_joint(const JointLaunch &L, WsHeader *hdr, cudaStream_t strea
 }
 
 int joint_rows_per_group() { return kRB; }
+int joint_round() { return kRound; }
+int joint_combos() { return kCombos; }
 
 namespace {
 __global__ void barrier_timeout_kernel(WsHeader *hdr, unsigned expected) { grid_barrier(hdr, expected); }
