@@ -171,6 +171,45 @@ def test_joint_isolated(name, seed):
     assert not acc[others].any()
 
 
+@pytest.mark.parametrize("name,seed,q", [("small", 0, 0.5), ("small", 1, 0.3), ("small_w40_g16", 2, 0.6),
+                                         ("small_long_pages", 4, 0.5)])
+def test_joint_rounds_with_rejections(name, seed, q):
+    """Up to 23 candidates (several rounds of the joint kernel and a ragged
+    last one) with tau at a quantile of their single-page effects, so that
+    the scan accepts and rejects, also in the middle of a round; every step
+    against the oracle's greedy scan, up to the first decision inside the
+    tolerance."""
+    r = get_run(name, seed)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    Rp = o.R_post
+    pages = [E for E in np.argsort(Rp, kind="stable") if np.isfinite(Rp[E]) and Rp[E] > 0][:23]
+    rng = np.random.default_rng(seed)
+    cand_np = np.array(pages, np.int64)[rng.permutation(len(pages))]
+    tau = float(np.float32(np.quantile(Rp[cand_np], q)))
+    acc_o, step_o = core.greedy(o.post, cand_np, tau, "closed", stats=o.stats)
+    nc = len(cand_np)
+    assert 2 <= int(acc_o[cand_np].sum()) <= nc - 2, "the scan should both accept and reject"
+    b.score_post()
+    cand = torch.zeros(max(dev.P_post, 1), dtype=torch.int32, device="cuda")
+    cand[:nc] = torch.from_numpy(cand_np.astype(np.int32)).cuda()
+    n_cand = torch.tensor([nc], dtype=torch.int32, device="cuda")
+    ck.commitkv_joint_test(b.shape, [dev.post()], b.stats, [cand], n_cand, tau, b.accepted, b.step_R,
+                           workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    step = _np(b.step_R[0])[:nc]
+    acc = _np(b.accepted[0])[:dev.P_post]
+    safe = safe_threshold_mask(step_o, tau, r.tol)
+    upto = nc if safe.all() else int(np.argmin(safe))
+    _assert_close(step[:upto], step_o[:upto], r.tol, "joint step R")
+    for j in range(upto):
+        assert acc[cand_np[j]] == acc_o[cand_np[j]], (j, step[j], step_o[j])
+    for j in range(nc):
+        assert acc[cand_np[j]] == (step[j] <= tau)
+    others = np.setdiff1d(np.arange(dev.P_post), cand_np)
+    assert not acc[others].any()
+
+
 @pytest.mark.parametrize("name,seed", CASES)
 def test_compact_isolated(name, seed):
     """Same retired set, pending pages, priorities and fill scores into the
