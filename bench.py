@@ -33,6 +33,23 @@ import numpy as np  # noqa: E402
 
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu pass) of
+# one scoring call of a step (prep + pass A + combine + pass B over the pre-
+# and post-commit caches), full-size workload, with the sha256 prefix of the
+# scoring sources they were taken with: reported only while those sources are
+# unchanged.
+MEASURED_TRAFFIC = {"qwen3_8b_32k": (18979224320, "82c23e8c98cfc00b")}
+TRAFFIC_SOURCES = ("score_tc.cu", "score_tc.cuh", "sm103.cuh")
+
+
+def scoring_sources_sha() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in TRAFFIC_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_07855_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -46,7 +63,7 @@ def load_peaks():
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default="qwen3_8b_32k")
     ap.add_argument("--seed", type=int, default=0)
@@ -78,12 +95,21 @@ class Clocks:
         self.proc = None
 
     def start(self):
+        """Starts sampling every 100 ms and returns once the first sample is
+        in, so that the samples fall inside the timed region that follows."""
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+                 "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
+            return
+        t0 = time.time()
+        while time.time() - t0 < 3.0 and self.proc.poll() is None:
+            self.f.flush()
+            if os.path.getsize(self.f.name) > 0:
+                break
+            time.sleep(0.02)
 
     def stop(self):
         if self.proc is None:
@@ -251,6 +277,9 @@ def run_ours(args, rank, world, local):
                 "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["traffic"] = None
+    mt = MEASURED_TRAFFIC.get(cfg.name)
+    if mt and world == 1 and scoring_sources_sha() == mt[1]:
+        roof["traffic"] = mt[0]  # bytes per step, against algorithmic_bytes_per_step
     roof["kernel"] = "commitkv_page_effects (pre + post scoring passes)"
     roof["peak_source"] = f"{peak_kind} ({'MEASURED_PEAKS.json' if peak_kind == 'measured' else 'recipe fallback'})"
     roof["algorithmic_bytes_per_step"] = alg_bytes
