@@ -286,6 +286,22 @@ def run_ours(args, rank, world, local):
     roof["algorithmic_flops_per_step"] = alg_flops
     roof["scoring_ms_per_step"] = score_ms
 
+    # the one-read variant (row stats given, page pass only) on the post-commit
+    # caches with the step's own stats: a side figure, not part of the step
+    single = None
+    if world == 1:
+        posts = [t.post() for t in buf.trajs]
+        for _ in range(2):
+            ck.commitkv_page_effects_from_stats(buf.shape, posts, buf.stats, buf.R_post, workspace=buf.ws)
+        a = torch.cuda.Event(enable_timing=True)
+        b_ = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(10):
+            ck.commitkv_page_effects_from_stats(buf.shape, posts, buf.stats, buf.R_post, workspace=buf.ws)
+        b_.record(stream)
+        torch.cuda.synchronize()
+        single = sum(t.S_post for t in trs) / (a.elapsed_time(b_) / 10 / 1e3)
+
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -303,6 +319,7 @@ def run_ours(args, rank, world, local):
                    "l2": "inputs larger than L2 (no flush)", "parallelism": f"replicas x{world}"},
         "stage_ms": stage_ms,
         "scoring_tokens_per_s": tokens_per_step * world / (score_ms / 1e3),
+        "single_read_scoring_tokens_per_s": single,
         "roofline": roof,
         "clocks": clk,
         "gpu_launches": buf_launches(buf) * args.steps,

@@ -177,6 +177,36 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
                                       size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Page deletion effects from given row statistics (Section 3.2, Eq. 6-8),
+ * one read of the page tokens.
+ *
+ * Eq. 6 needs, per probe row, the final softmax of the whole cache: the
+ * normaliser and the output o_p.  An engine that already computed that
+ * attention (its output and log-sum-exp for the probe queries) can pass
+ * them here; the library then reads only the tokens of the pages (one pass)
+ * instead of the whole cache and then the pages (two passes, as
+ * commitkv_page_effects does).  Same definition, same degenerate cases and
+ * same outputs as commitkv_page_effects.
+ *
+ *   stats_in     host array [n_traj] of device float [M][Hq][W_t][d + 4]
+ *                (entries of trajectories with P = 0 or W = 0 may be NULL):
+ *                per probe row m, l, (ignored), (ignored), o_p[0..d) with
+ *                l = sum over visible i of exp(softmax_scale <q_p, k_i> - m)
+ *                and o_p the normalised output.  From a log-sum-exp L: m = L,
+ *                l = 1.  The stats_out of commitkv_page_effects on the same
+ *                cache and window are valid stats_in.  Rows of unselected
+ *                layers are not read.  Read only.
+ *   R_out, head_R_out, layer_mask   as for commitkv_page_effects.
+ * The number of visible tokens of each row is counted from pos and q_pos.
+ * A row whose stats disagree with its cache gives effects of those stats.
+ * -------------------------------------------------------------------- */
+commitkv_status commitkv_page_effects_from_stats(const commitkv_shape *shape, int32_t n_traj,
+                                                 const commitkv_traj *trajs, const uint8_t *layer_mask,
+                                                 const float *const *stats_in, float *const *R_out,
+                                                 float *const *head_R_out, void *workspace,
+                                                 size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Lifecycle classification, Section 3.3, Eq. 9-10, and the candidate order
  * of Section 3.4.
  *

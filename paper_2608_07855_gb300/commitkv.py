@@ -85,6 +85,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.commitkv_status_string.argtypes = [ctypes.c_int]
     lib.commitkv_status_string.restype = ctypes.c_char_p
     lib.commitkv_page_effects.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, sz, vp]
+    lib.commitkv_page_effects_from_stats.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, sz, vp]
     lib.commitkv_classify.argtypes = [i32, vp, vp, vp, vp, P(Thresholds), vp, vp, vp, vp, sz, vp]
     lib.commitkv_joint_test.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, ctypes.c_float,
                                         vp, vp, vp, sz, vp]
@@ -94,7 +95,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
                                              i32, vp, vp, vp, vp, vp, vp, vp]
     lib.commitkv_test_barrier_timeout.argtypes = [vp, sz, i32, vp]
     for f in ("commitkv_workspace_init", "commitkv_workspace_status", "commitkv_page_effects",
-              "commitkv_classify", "commitkv_joint_test", "commitkv_compact",
+              "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_joint_test", "commitkv_compact",
               "commitkv_compact_noalloc", "commitkv_test_barrier_timeout"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
@@ -264,6 +265,18 @@ def commitkv_page_effects(shape: Shape, trajs, R_out, head_R_out=None, stats_out
         ctypes.byref(shape), n, d, mptr, _ptr_array(R_out, n), _ptr_array(head_R_out, n),
         _ptr_array(stats_out, n), _ptr(workspace), workspace.numel(), _stream(stream))
     _check(rc, "commitkv_page_effects")
+
+
+def commitkv_page_effects_from_stats(shape: Shape, trajs, stats_in, R_out, head_R_out=None,
+                                     layer_mask=None, workspace=None, stream=None):
+    n = len(trajs)
+    d = _descs(trajs)
+    _mbuf, mptr = _mask(layer_mask, shape.layers)
+    _require_cuda(*R_out)
+    rc = load_library().commitkv_page_effects_from_stats(
+        ctypes.byref(shape), n, d, mptr, _ptr_array(stats_in, n), _ptr_array(R_out, n),
+        _ptr_array(head_R_out, n), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(rc, "commitkv_page_effects_from_stats")
 
 
 def commitkv_classify(P, R_pre, R_post, eligible, state_out, cand_out, n_cand_out, workspace,

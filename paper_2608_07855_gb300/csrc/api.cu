@@ -173,7 +173,7 @@ size_t score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr,
   for (int t = 0; t < n_traj; ++t) {
     int rows = g * tr[t].W;
     units += (size_t)n_layers * s->kv_heads * simt_chunk_bound(tr[t].S) * cdiv(rows, RB);
-    stats += align_up((size_t)s->layers * s->q_heads * tr[t].W * (d + 4) * 4);
+    stats += align_up((size_t)s->layers * s->q_heads * tr[t].W * (d + 4) * 4) + align_up((size_t)tr[t].W * 4);
   }
   size_t scratch = align_up(units * RB * (d + 4) * 4);
   if (s->head_dim == 128) {
@@ -269,17 +269,23 @@ const char *commitkv_status_string(commitkv_status s) {
   return "unknown status";
 }
 
-commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_traj,
-                                      const commitkv_traj *trajs, const uint8_t *layer_mask,
-                                      float *const *R_out, float *const *head_R_out,
-                                      float *const *stats_out, void *workspace,
-                                      size_t workspace_bytes, cudaStream_t stream) {
+namespace {
+
+// Scoring of both entry points: with stats_in the row stats are the
+// caller's and only the page pass runs.
+commitkv_status page_effects_impl(const commitkv_shape *shape, int32_t n_traj, const commitkv_traj *trajs,
+                                  const uint8_t *layer_mask, const float *const *stats_in,
+                                  float *const *R_out, float *const *head_R_out, float *const *stats_out,
+                                  void *workspace, size_t workspace_bytes, cudaStream_t stream) {
   commitkv_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_trajs(shape, n_traj, trajs, true))) return st;
   if (!R_out) return COMMITKV_ERR_INVALID_ARG;
-  for (int t = 0; t < n_traj; ++t)
+  for (int t = 0; t < n_traj; ++t) {
     if (trajs[t].P > 0 && !R_out[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (stats_in && trajs[t].P > 0 && trajs[t].W > 0 && !stats_in[t]) return COMMITKV_ERR_INVALID_ARG;
+  }
+  const bool from_stats = stats_in != nullptr;
 
   static thread_local ScoreLaunch L;  // large: keep off the stack
   memset(&L, 0, sizeof L);
@@ -317,11 +323,17 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
   char *sbase = base + scratch;
   for (int t = 0; t < n_traj; ++t) {
     size_t sb = align_up((size_t)shape->layers * shape->q_heads * trajs[t].W * (d + 4) * 4);
-    L.stats[t] = (stats_out && stats_out[t]) ? stats_out[t] : reinterpret_cast<float *>(sbase);
+    if (from_stats) L.stats[t] = const_cast<float *>(stats_in[t]);  // read only
+    else L.stats[t] = (stats_out && stats_out[t]) ? stats_out[t] : reinterpret_cast<float *>(sbase);
     sbase += sb;
     L.R[t] = R_out[t];
     L.headR[t] = head_R_out ? head_R_out[t] : nullptr;
   }
+  for (int t = 0; t < n_traj; ++t) {
+    L.nvis_w[t] = reinterpret_cast<int32_t *>(sbase);
+    sbase += align_up((size_t)trajs[t].W * 4);
+  }
+  L.from_stats = from_stats ? 1 : 0;
   for (int t = 0; t < n_traj; ++t) {
     if (trajs[t].P == 0) continue;
     cudaError_t e = cudaMemsetAsync(R_out[t], 0, (size_t)trajs[t].P * 4, stream);
@@ -356,6 +368,7 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
     T.n_layers = nl;
     T.chunk_len = CLt;
     T.slots_per_item = tc::kSlotsPerItem;
+    T.from_stats = L.from_stats;
     T.scale_log2 = L.batch.scale_log2;
     T.partials = tc_partials;
     memcpy(T.layer_ids, L.batch.layer_ids, sizeof T.layer_ids);
@@ -377,6 +390,7 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
       tt.slot_tab = reinterpret_cast<int4 *>(slot_base);
       slot_base += align_up(((size_t)cdiv(x.S, 16) + x.P) * 16);
       tt.stats = L.stats[t];
+      tt.nvis_w = L.nvis_w[t];
       tt.R = L.R[t];
       tt.headR = L.headR[t];
       tt.S = x.S;
@@ -398,6 +412,27 @@ commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_tra
     if (e != cudaSuccess) return cuda_status(e);
   }
   return COMMITKV_OK;
+}
+
+}  // namespace
+
+commitkv_status commitkv_page_effects(const commitkv_shape *shape, int32_t n_traj,
+                                      const commitkv_traj *trajs, const uint8_t *layer_mask,
+                                      float *const *R_out, float *const *head_R_out,
+                                      float *const *stats_out, void *workspace,
+                                      size_t workspace_bytes, cudaStream_t stream) {
+  return page_effects_impl(shape, n_traj, trajs, layer_mask, nullptr, R_out, head_R_out, stats_out, workspace,
+                           workspace_bytes, stream);
+}
+
+commitkv_status commitkv_page_effects_from_stats(const commitkv_shape *shape, int32_t n_traj,
+                                                 const commitkv_traj *trajs, const uint8_t *layer_mask,
+                                                 const float *const *stats_in, float *const *R_out,
+                                                 float *const *head_R_out, void *workspace,
+                                                 size_t workspace_bytes, cudaStream_t stream) {
+  if (!stats_in) return COMMITKV_ERR_INVALID_ARG;
+  return page_effects_impl(shape, n_traj, trajs, layer_mask, stats_in, R_out, head_R_out, nullptr, workspace,
+                           workspace_bytes, stream);
 }
 
 commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float *const *R_pre,

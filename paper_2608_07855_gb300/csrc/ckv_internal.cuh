@@ -110,6 +110,8 @@ struct ScoreLaunch {
   float *stats[kMaxTraj];            // [M][Hq][W][d + 4]
   float *R[kMaxTraj];
   float *headR[kMaxTraj];
+  int32_t *nvis_w[kMaxTraj];         // [W]: resident tokens visible to each window position
+  int32_t from_stats;                // the stats are the caller's: no flash pass, no combine
 };
 
 cudaError_t launch_score_simt(const ScoreLaunch &L, float *partials, WsHeader *hdr,

@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(kThreads) pass_b_kernel(const __grid_constant_
     float mn = ok ? st[0] : kNegInf;
     m2[k] = mn == kNegInf ? mn : mn * 1.4426950408889634f;
     lsum[k] = ok ? st[1] : 0.0f;
-    nvis[k] = ok ? (int)st[2] : 0;
+    nvis[k] = ok ? L.nvis_w[t][w] : 0;
     qp[k] = ok ? tr.qpos[w] : -0x7fffffff;
     float ss = 0.0f;
 #pragma unroll
@@ -341,6 +341,23 @@ __global__ void __launch_bounds__(kThreads) pass_b_kernel(const __grid_constant_
   for (int E = E0 + threadIdx.x; E < E1; E += kThreads) atomic_max_nonneg(L.R[t] + E, sR[E - E0]);
 }
 
+// Per trajectory and window position w: the number of resident tokens with
+// pos <= qpos[w] (positions increase, so a binary search).
+__global__ void __launch_bounds__(256) count_visible_kernel(const __grid_constant__ ScoreLaunch L) {
+  const int t = blockIdx.x;
+  const TrajDev &tr = L.batch.t[t];
+  for (int w = threadIdx.x; w < tr.W; w += blockDim.x) {
+    const int qp = tr.qpos[w];
+    int a = 0, b = tr.S;
+    while (a < b) {
+      int mid = (a + b) >> 1;
+      if (tr.pos[mid] <= qp) a = mid + 1;
+      else b = mid;
+    }
+    L.nvis_w[t][w] = a;
+  }
+}
+
 template <typename T, int D>
 cudaError_t launch_typed(const ScoreLaunch &L, float *partials, WsHeader *hdr, cudaStream_t s) {
   size_t smem = (size_t)(kRB * D + kTK * (D + 1) + kTK * D) * 4 + kTK * 4 + kWarps * kTK * 4 + kPG * 4;
@@ -349,9 +366,10 @@ cudaError_t launch_typed(const ScoreLaunch &L, float *partials, WsHeader *hdr, c
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(pass_b_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  int na = L.unit_off_a[L.batch.n_traj];
+  count_visible_kernel<<<L.batch.n_traj, 256, 0, s>>>(L);
+  int na = L.from_stats ? 0 : L.unit_off_a[L.batch.n_traj];
   if (na > 0) pass_a_kernel<T, D><<<na, kThreads, smem, s>>>(L, partials);
-  int rows = L.row_off[L.batch.n_traj];
+  int rows = L.from_stats ? 0 : L.row_off[L.batch.n_traj];
   if (rows > 0) combine_kernel<D><<<(rows * 32 + kThreads - 1) / kThreads, kThreads, 0, s>>>(L, partials);
   int nb = L.unit_off_b[L.batch.n_traj];
   if (nb > 0) pass_b_kernel<T, D><<<nb, kThreads, smem, s>>>(L, hdr);

@@ -536,7 +536,8 @@ __global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaun
 //   the pass-B work items: item k takes the pages whose first slot lies in
 //   [k * slots_per_item, (k + 1) * slots_per_item);
 //   vis_all = number of leading resident tokens visible to every probe row
-//   (positions increase, so this is a prefix).
+//   (positions increase, so this is a prefix); nvis_w[w] = number of resident
+//   tokens visible to window position w.
 __global__ void __launch_bounds__(1024) prep_kernel(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
   const TcTraj &tr = L.t[blockIdx.x];
   int lane = threadIdx.x % 32, wid = threadIdx.x / 32;
@@ -611,6 +612,16 @@ __global__ void __launch_bounds__(1024) prep_kernel(const __grid_constant__ TcLa
     for (int E = E0; E < E1; ++E) npages += tr.slot_off[E + 1] > tr.slot_off[E];
     tr.items[2 * k] = make_int4(E0, E1, slot0, nslot);
     tr.items[2 * k + 1] = make_int4(npages, 0, 0, 0);
+  }
+  for (int w = threadIdx.x; w < tr.W; w += blockDim.x) {
+    const int qp = tr.qpos[w];
+    int a = 0, b = tr.S;
+    while (a < b) {
+      int mid = (a + b) >> 1;
+      if (tr.pos[mid] <= qp) a = mid + 1;
+      else b = mid;
+    }
+    tr.nvis_w[w] = a;
   }
   if (threadIdx.x == 0) {
     int qmin = 0x7fffffff;
@@ -1092,7 +1103,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
         const float *st = tr.stats + (((int64_t)bi.l * L.Hq + h) * tr.W + w) * (D + 4);
         float4 hd = valid_row ? *reinterpret_cast<const float4 *>(st) : make_float4(0.f, 0.f, 0.f, 0.f);
         lsum = hd.y;
-        nvis = (int)hd.z;
+        nvis = valid_row ? tr.nvis_w[w] : 0;
         float ss = 0.0f;
 #pragma unroll
         for (int c = 0; c < D; c += 4) {
@@ -1216,9 +1227,9 @@ cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, in
   e = cudaFuncSetAttribute(pass_b_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_b());
   if (e != cudaSuccess) return e;
   prep_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
-  int na = L.item_off_a[L.n_traj];
+  int na = L.from_stats ? 0 : L.item_off_a[L.n_traj];
   if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 384, smem_a(), s>>>(L, hdr);
-  int rows = L.row_off[L.n_traj];
+  int rows = L.from_stats ? 0 : L.row_off[L.n_traj];
   if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
   int nb = L.item_off_b[L.n_traj];
   if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 512, smem_b(), s>>>(L, hdr);

@@ -31,6 +31,7 @@ struct TcTraj {
   int4 *items;        // workspace [nbitem][2]: {E0, E1, slot0, nslot}, {npages, 0, 0, 0}
   int4 *slot_tab;     // workspace [ceil(S/16) + P]: {tok0, nv, page, first | last << 1 | rank << 2}
   TcPrep *prep;       // workspace
+  int32_t *nvis_w;    // workspace [W]: resident tokens visible to each window position
   float *stats;       // [M][Hq][W][132]
   float *R;           // [P]
   float *headR;       // [M][Hq][P] or null
@@ -41,6 +42,7 @@ struct TcLaunch {
   TcMaps maps[kMaxTc];
   TcTraj t[kMaxTc];
   int n_traj, M, H, Hq, g, n_layers, chunk_len, slots_per_item;
+  int from_stats;  // the stats are the caller's: no flash pass, no combine
   float scale_log2;
   float *partials;  // [items_a][2][128][132]: one partial per softmax warpgroup
   int item_off_a[kMaxTc + 1], item_off_b[kMaxTc + 1], row_off[kMaxTc + 1];

@@ -318,6 +318,56 @@ def test_batched_trajectories_match_single():
         _assert_close(_np(Rp), o.R_post, 2e-2, "batched R+")
 
 
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("small", 0), ("small_w40_g16", 2), ("small_long_pages", 4),
+                                       ("small_f32", 3)])
+def test_from_stats_matches_full_call(name, seed):
+    """The page pass alone, fed the stats the full call wrote, gives the
+    same effects bit for bit (both paths: the CUDA-core one for fp32 and
+    head width 64, the tensor-core one for bf16)."""
+    r = get_run(name, seed)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    R = torch.zeros(dev.P_post, device="cuda")
+    H = torch.zeros(cfg.M, cfg.Hq, dev.P_post, device="cuda")
+    st = torch.zeros_like(b.stats[0])
+    ck.commitkv_page_effects(b.shape, [dev.post()], [R], head_R_out=[H], stats_out=[st], workspace=b.ws)
+    R2 = torch.full_like(R, 7.0)
+    H2 = torch.full_like(H, 7.0)
+    ck.commitkv_page_effects_from_stats(b.shape, [dev.post()], [st], [R2], head_R_out=[H2], workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    assert torch.equal(R.view(torch.int32), R2.view(torch.int32))
+    assert torch.equal(H.view(torch.int32), H2.view(torch.int32))
+
+
+def _oracle_stats(cfg, o, lse_form):
+    m, l, o_vec, n = o.stats
+    st = np.zeros((cfg.M * cfg.Hq * o.tr.cfg.W, cfg.d + 4))
+    if lse_form:  # an engine's log-sum-exp: m = L, l = 1
+        st[:, 0] = np.where(np.isfinite(m), m + np.log(np.where(l > 0, l, 1.0)), m)
+        st[:, 1] = np.where(np.isfinite(m), 1.0, 0.0)
+    else:
+        st[:, 0], st[:, 1] = m, l
+    st[:, 4:] = o_vec
+    return torch.from_numpy(st.astype(np.float32).reshape(cfg.M, cfg.Hq, o.tr.cfg.W, cfg.d + 4)).cuda()
+
+
+@pytest.mark.parametrize("name,seed", [("tiny", 1), ("small", 1), ("small_long_pages", 4)])
+@pytest.mark.parametrize("lse_form", [False, True])
+def test_from_stats_with_oracle_stats(name, seed, lse_form):
+    """The oracle's fp64 row stats (rounded to fp32), as (max, sum) or as a
+    log-sum-exp with sum 1, into the page pass: effects against the oracle."""
+    r = get_run(name, seed)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    st = _oracle_stats(cfg, o, lse_form)
+    R = torch.zeros(dev.P_post, device="cuda")
+    H = torch.zeros(cfg.M, cfg.Hq, dev.P_post, device="cuda")
+    ck.commitkv_page_effects_from_stats(b.shape, [dev.post()], [st], [R], head_R_out=[H], workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    _assert_close(_np(R), o.R_post, r.tol, "R+ from oracle stats")
+    _assert_close(_np(H), o.H_post, r.tol, "R+ per head from oracle stats")
+
+
 def test_pre_and_post_in_one_call():
     """The pre- and post-commit caches of three trajectories scored in one
     call (six caches in one launch sequence): effects match the oracle and
