@@ -235,6 +235,35 @@ commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float 
                                   size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Classification variants: the ablations of Section 4.4 (Table 3).
+ *
+ * commitkv_classify with some of its steps removed; variant = 0 is
+ * commitkv_classify.  Bits:
+ *   COMMITKV_CLASSIFY_NO_PRECOMMIT   "w/o pre-commit state": the candidates
+ *       are the pages with L+ (low after the commit) whatever their state
+ *       before it, instead of H- and L+.  state_out is still the lifecycle
+ *       state of Eq. 10; cand_out / n_cand_out list the L+ pages in the
+ *       same order (increasing R+, then decreasing R-, then page index).
+ *   COMMITKV_CLASSIFY_NO_PERCENTILE  "w/o percentile calibration": H = (R >=
+ *       tau_use) and L = (R <= tau_dead) in both windows; rho_use and
+ *       rho_dead are not used (they are still checked).
+ * The paper's other ablations need no variant: "w/o joint validation"
+ * retires every candidate (commitkv_joint_test with tau_joint = +inf),
+ * "w/o transition protection" reserves no pending pages
+ * (commitkv_compact with pending_cap_pages = 0), "w/o lifecycle mechanism"
+ * retires nothing (no classify and joint test before commitkv_compact).
+ * Unknown bits: COMMITKV_ERR_INVALID_ARG.  Otherwise as commitkv_classify.
+ * -------------------------------------------------------------------- */
+#define COMMITKV_CLASSIFY_NO_PRECOMMIT 1u
+#define COMMITKV_CLASSIFY_NO_PERCENTILE 2u
+commitkv_status commitkv_classify_variant(int32_t n_traj, const int32_t *P, const float *const *R_pre,
+                                          const float *const *R_post, const uint8_t *const *eligible,
+                                          const commitkv_thresholds *thresholds, uint32_t variant,
+                                          uint8_t *const *state_out, int32_t *const *cand_out,
+                                          int32_t *n_cand_out, void *workspace, size_t workspace_bytes,
+                                          cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Greedy joint test, Section 3.4, Eq. 11 and the inner loop of Algorithm 1.
  *
  * Per trajectory, with A = {} and the candidates in the order given:

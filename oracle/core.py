@@ -220,13 +220,19 @@ def percentile_ranks(R, idx) -> np.ndarray:
     return k / float(n) if n else np.zeros(0)
 
 
-def classify(R_pre, R_post, eligible, tau_use=0.05, tau_dead=0.01, rho_use=0.75, rho_dead=0.25):
+def classify(R_pre, R_post, eligible, tau_use=0.05, tau_dead=0.01, rho_use=0.75, rho_dead=0.25,
+             no_precommit=False, no_percentile=False):
     """Lifecycle states of Eq. 10 and the ordered completion candidates.
 
     eligible marks E_c, the pages measurable in both windows.  States:
     STATE_NONE outside E_c, else candidate / dormant / newly active /
     still active / uncertain.  Candidates are ordered by increasing R+,
-    then decreasing R-, then increasing page index."""
+    then decreasing R-, then increasing page index.
+
+    The ablations of Section 4.4: no_percentile drops the percentile
+    conditions from H and L (absolute thresholds only); no_precommit takes
+    as candidates every page with L+ instead of H- and L+ (the states are
+    unchanged)."""
     R_pre = np.asarray(R_pre, np.float64)
     R_post = np.asarray(R_post, np.float64)
     P = R_pre.shape[0]
@@ -243,6 +249,10 @@ def classify(R_pre, R_post, eligible, tau_use=0.05, tau_dead=0.01, rho_use=0.75,
     Pm = percentile_ranks(R_pre, idx)
     Pp = percentile_ranks(R_post, idx)
     Rm, Rp = R_pre[idx], R_post[idx]
+    if no_percentile:
+        Pm = np.full(len(idx), 0.5)  # inside every percentile condition below
+        Pp = np.full(len(idx), 0.5)
+        r_use, r_dead = 0.0, 1.0
     Hm = (Rm >= t_use) & (Pm >= r_use)
     Lm = (Rm <= t_dead) & (Pm <= r_dead)
     Hp = (Rp >= t_use) & (Pp >= r_use)
@@ -253,7 +263,7 @@ def classify(R_pre, R_post, eligible, tau_use=0.05, tau_dead=0.01, rho_use=0.75,
     st[Lm & Hp] = STATE_NEWLY_ACTIVE
     st[Hm & Hp] = STATE_STILL_ACTIVE
     state[idx] = st
-    cand = idx[st == STATE_CANDIDATE]
+    cand = idx[Lp] if no_precommit else idx[st == STATE_CANDIDATE]
     order = sorted(cand.tolist(), key=lambda E: (R_post[E], -R_pre[E], E))
     return state, np.asarray(order, np.int32)
 

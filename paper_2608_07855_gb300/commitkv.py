@@ -87,6 +87,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.commitkv_page_effects.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, sz, vp]
     lib.commitkv_page_effects_from_stats.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, sz, vp]
     lib.commitkv_classify.argtypes = [i32, vp, vp, vp, vp, P(Thresholds), vp, vp, vp, vp, sz, vp]
+    lib.commitkv_classify_variant.argtypes = [i32, vp, vp, vp, vp, P(Thresholds), ctypes.c_uint32, vp, vp, vp,
+                                              vp, sz, vp]
     lib.commitkv_joint_test.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, ctypes.c_float,
                                         vp, vp, vp, sz, vp]
     lib.commitkv_compact.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, i32, i32, i32,
@@ -95,7 +97,7 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
                                              i32, vp, vp, vp, vp, vp, vp, vp]
     lib.commitkv_test_barrier_timeout.argtypes = [vp, sz, i32, vp]
     for f in ("commitkv_workspace_init", "commitkv_workspace_status", "commitkv_page_effects",
-              "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_joint_test", "commitkv_compact",
+              "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_classify_variant", "commitkv_joint_test", "commitkv_compact",
               "commitkv_compact_noalloc", "commitkv_test_barrier_timeout"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
@@ -289,6 +291,22 @@ def commitkv_classify(P, R_pre, R_post, eligible, state_out, cand_out, n_cand_ou
         _ptr_array(state_out, n), _ptr_array(cand_out, n), _ptr(n_cand_out), _ptr(workspace),
         workspace.numel(), _stream(stream))
     _check(rc, "commitkv_classify")
+
+
+COMMITKV_CLASSIFY_NO_PRECOMMIT = 1
+COMMITKV_CLASSIFY_NO_PERCENTILE = 2
+
+
+def commitkv_classify_variant(P, R_pre, R_post, eligible, variant, state_out, cand_out, n_cand_out,
+                              workspace, thresholds: Optional[Thresholds] = None, stream=None):
+    n = len(P)
+    Parr = (ctypes.c_int32 * n)(*[int(p) for p in P])
+    rc = load_library().commitkv_classify_variant(
+        n, ctypes.cast(Parr, ctypes.c_void_p), _ptr_array(R_pre, n), _ptr_array(R_post, n),
+        _ptr_array(eligible, n), ctypes.byref(thresholds) if thresholds else None, int(variant),
+        _ptr_array(state_out, n), _ptr_array(cand_out, n), _ptr(n_cand_out), _ptr(workspace),
+        workspace.numel(), _stream(stream))
+    _check(rc, "commitkv_classify_variant")
 
 
 def commitkv_joint_test(shape: Shape, post, stats, cand, n_cand, tau_joint, accepted_out,

@@ -440,8 +440,20 @@ commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float 
                                   const commitkv_thresholds *thresholds, uint8_t *const *state_out,
                                   int32_t *const *cand_out, int32_t *n_cand_out, void *workspace,
                                   size_t workspace_bytes, cudaStream_t stream) {
+  return commitkv_classify_variant(n_traj, P, R_pre, R_post, eligible, thresholds, 0u, state_out, cand_out,
+                                   n_cand_out, workspace, workspace_bytes, stream);
+}
+
+commitkv_status commitkv_classify_variant(int32_t n_traj, const int32_t *P, const float *const *R_pre,
+                                          const float *const *R_post, const uint8_t *const *eligible,
+                                          const commitkv_thresholds *thresholds, uint32_t variant,
+                                          uint8_t *const *state_out, int32_t *const *cand_out,
+                                          int32_t *n_cand_out, void *workspace, size_t workspace_bytes,
+                                          cudaStream_t stream) {
   if (n_traj < 1 || n_traj > kMaxTraj || !P || !R_pre || !R_post || !eligible || !state_out ||
       !cand_out || !n_cand_out)
+    return COMMITKV_ERR_INVALID_ARG;
+  if (variant & ~(uint32_t)(COMMITKV_CLASSIFY_NO_PRECOMMIT | COMMITKV_CLASSIFY_NO_PERCENTILE))
     return COMMITKV_ERR_INVALID_ARG;
   commitkv_thresholds th = thresholds ? *thresholds : commitkv_thresholds{0.05f, 0.01f, 0.75f, 0.25f};
   if (!(th.tau_dead < th.tau_use) || !(th.rho_dead < th.rho_use)) return COMMITKV_ERR_INVALID_ARG;
@@ -471,6 +483,7 @@ commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float 
   L.tau_dead = th.tau_dead;
   L.rho_use = (double)th.rho_use;
   L.rho_dead = (double)th.rho_dead;
+  L.variant = variant;
   return cuda_status(launch_classify(L, static_cast<WsHeader *>(workspace), stream));
 }
 

@@ -129,6 +129,7 @@ struct ClassifyLaunch {
   int32_t *n_cand;
   float tau_use, tau_dead;
   double rho_use, rho_dead;
+  uint32_t variant;  // COMMITKV_CLASSIFY_NO_* bits (the ablations of Section 4.4)
 };
 cudaError_t launch_classify(const ClassifyLaunch &L, WsHeader *hdr, cudaStream_t stream);
 

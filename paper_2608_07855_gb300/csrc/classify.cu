@@ -57,17 +57,21 @@ __global__ void __launch_bounds__(kThreads) classify_kernel(const __grid_constan
       kp += Rp[F] < rp;
     }
     double Pm = (double)km / (double)n, Pp = (double)kp / (double)n;
-    bool Hm = rm >= L.tau_use && Pm >= L.rho_use;
-    bool Lm = rm <= L.tau_dead && Pm <= L.rho_dead;
-    bool Hp = rp >= L.tau_use && Pp >= L.rho_use;
-    bool Lp = rp <= L.tau_dead && Pp <= L.rho_dead;
+    // without percentile calibration the states use the absolute thresholds only
+    const bool pct = !(L.variant & COMMITKV_CLASSIFY_NO_PERCENTILE);
+    bool Hm = rm >= L.tau_use && (!pct || Pm >= L.rho_use);
+    bool Lm = rm <= L.tau_dead && (!pct || Pm <= L.rho_dead);
+    bool Hp = rp >= L.tau_use && (!pct || Pp >= L.rho_use);
+    bool Lp = rp <= L.tau_dead && (!pct || Pp <= L.rho_dead);
     uint8_t st = 5;  // uncertain
     if (Hm && Lp) st = 1;       // completion candidate
     else if (Lm && Lp) st = 2;  // dormant
     else if (Lm && Hp) st = 3;  // newly active
     else if (Hm && Hp) st = 4;  // still active
     L.state[t][E] = st;
-    if (st == 1) L.scratch[t][atomicAdd(&s_c, 1)] = E;
+    // without the pre-commit state every page low after the commit is a candidate
+    const bool cand = (L.variant & COMMITKV_CLASSIFY_NO_PRECOMMIT) ? Lp : st == 1;
+    if (cand) L.scratch[t][atomicAdd(&s_c, 1)] = E;
   }
   __syncthreads();
   int C = s_c;

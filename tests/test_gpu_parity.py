@@ -138,6 +138,43 @@ def test_classify_isolated(name, seed):
     assert np.array_equal(_np(b.cand[0])[:nc], o.cand)
 
 
+@pytest.mark.parametrize("variant", [1, 2, 3])
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("small", 1), ("small_w40_g16", 2), ("hand", 0)])
+def test_classify_variants(name, seed, variant):
+    """The ablations of Section 4.4 (w/o pre-commit state, w/o percentile
+    calibration, both): states and candidate order bit for bit against the
+    oracle on the same fp32 effects."""
+    import json
+    import os
+    np_ = ck.COMMITKV_CLASSIFY_NO_PRECOMMIT & variant != 0
+    npc = ck.COMMITKV_CLASSIFY_NO_PERCENTILE & variant != 0
+    if name == "hand":
+        with open(os.path.join(os.path.dirname(__file__), "golden", "classify_variants_hand.json")) as f:
+            g = json.load(f)
+        Rm32 = np.asarray(g["R_pre"], np.float32)
+        Rp32 = np.asarray(g["R_post"], np.float32)
+        el = torch.tensor(g["eligible"], dtype=torch.uint8, device="cuda")
+        ws = get_run("small", 0).buf.ws  # sized for far more than 8 pages
+    else:
+        r = get_run(name, seed)
+        Rm32, Rp32 = r.orc.R_pre32, r.orc.R_post32
+        el = r.dev.eligible
+        ws = r.buf.ws
+    P = len(Rm32)
+    st_o, cand_o = core.classify(Rm32, Rp32, _np(el), no_precommit=np_, no_percentile=npc)
+    state = torch.zeros(max(P, 1), dtype=torch.uint8, device="cuda")
+    cand = torch.full((max(P, 1),), -1, dtype=torch.int32, device="cuda")
+    n_cand = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ck.commitkv_classify_variant([P], [torch.from_numpy(Rm32).cuda()], [torch.from_numpy(Rp32).cuda()], [el],
+                                 variant, [state], [cand], n_cand, ws)
+    torch.cuda.synchronize()
+    assert ck.commitkv_workspace_status(ws) == ck.COMMITKV_OK
+    assert np.array_equal(_np(state)[:P], st_o)
+    nc = int(n_cand[0])
+    assert nc == len(cand_o)
+    assert np.array_equal(_np(cand)[:nc], cand_o)
+
+
 @pytest.mark.parametrize("name,seed", CASES)
 def test_joint_isolated(name, seed):
     """The oracle's candidate list into the GPU joint test (with the GPU's
@@ -208,6 +245,31 @@ def test_joint_rounds_with_rejections(name, seed, q):
         assert acc[cand_np[j]] == (step[j] <= tau)
     others = np.setdiff1d(np.arange(dev.P_post), cand_np)
     assert not acc[others].any()
+
+
+def test_joint_without_validation_accepts_every_candidate():
+    """'w/o joint validation' (Section 4.4) is the joint test with tau_joint =
+    +inf: every candidate is retired; the step values are those of the scan
+    that accepts them all, against the oracle."""
+    r = get_run("small", 0)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    Rp = o.R_post
+    cand_np = np.array([E for E in np.argsort(Rp, kind="stable") if np.isfinite(Rp[E]) and Rp[E] > 0][:10], np.int64)
+    nc = len(cand_np)
+    acc_o, step_o = core.greedy(o.post, cand_np, float("inf"), "closed", stats=o.stats)
+    assert acc_o[cand_np].all()
+    b.score_post()
+    cand = torch.zeros(max(dev.P_post, 1), dtype=torch.int32, device="cuda")
+    cand[:nc] = torch.from_numpy(cand_np.astype(np.int32)).cuda()
+    n_cand = torch.tensor([nc], dtype=torch.int32, device="cuda")
+    ck.commitkv_joint_test(b.shape, [dev.post()], b.stats, [cand], n_cand, float("inf"), b.accepted, b.step_R,
+                           workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    acc = _np(b.accepted[0])[:dev.P_post]
+    assert acc[cand_np].all() and acc.sum() == nc
+    fin = np.isfinite(step_o)
+    _assert_close(_np(b.step_R[0])[:nc][fin], step_o[fin], r.tol, "step R with every candidate accepted")
 
 
 @pytest.mark.parametrize("name,seed", CASES)

@@ -240,6 +240,17 @@ def test_classify_hand(golden_dir):
         assert cand.tolist() == c["cand"], c["name"]
 
 
+def test_classify_variants_hand(golden_dir):
+    """The ablations of Section 4.4 on a hand-worked table."""
+    with open(os.path.join(golden_dir, "classify_variants_hand.json")) as f:
+        g = json.load(f)
+    for c in g["cases"]:
+        st, cand = core.classify(g["R_pre"], g["R_post"], g["eligible"], **g["thresholds"],
+                                 no_precommit=c["no_precommit"], no_percentile=c["no_percentile"])
+        assert st.tolist() == c["state"], c["name"]
+        assert cand.tolist() == c["cand"], c["name"]
+
+
 @pytest.mark.parametrize("seed", range(5))
 def test_classify_properties(seed):
     rng = np.random.default_rng(seed)
