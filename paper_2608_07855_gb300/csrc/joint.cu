@@ -267,17 +267,14 @@ __global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constan
           const int nt = min(kTK, ps + pl - tok0);
           __syncthreads();
           constexpr int V8 = 16 / sizeof(T);  // elements per 16-byte load
-          for (int e = threadIdx.x; e < kTK * D / V8; e += kThreads) {
+          // only the chunk's nt rows: the scores of the other rows are masked
+          // out below and P V stops at nt
+          for (int e = threadIdx.x; e < nt * (D / V8); e += kThreads) {
             const int i = e / (D / V8), ch = (e % (D / V8)) * V8;
             float kv[V8], vv[V8];
-            if (i < nt) {
-              const int64_t off = (int64_t)(tok0 + i) * tr.st + ch;
-              load16_f32<T>(kp + off, kv);
-              load16_f32<T>(vp + off, vv);
-            } else {
-#pragma unroll
-              for (int u = 0; u < V8; ++u) kv[u] = vv[u] = 0.0f;
-            }
+            const int64_t off = (int64_t)(tok0 + i) * tr.st + ch;
+            load16_f32<T>(kp + off, kv);
+            load16_f32<T>(vp + off, vv);
 #pragma unroll
             for (int u = 0; u < V8; u += 4) {
               *reinterpret_cast<float4 *>(sK + i * (D + 4) + ch + u) = make_float4(kv[u], kv[u + 1], kv[u + 2], kv[u + 3]);
@@ -293,6 +290,20 @@ __global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constan
 #pragma unroll
           for (int k = 0; k < kRowsPerWarp; ++k) s[k][0] = s[k][1] = 0.0f;
           const bool in0 = lane < nt, in1 = lane + 32 < nt;
+          if (nt <= 32) {  // one token per lane (warp-uniform)
+#pragma unroll 2
+            for (int ch = 0; ch < D; ch += 4) {
+              const float4 k0 = *reinterpret_cast<const float4 *>(sK + lane * (D + 4) + ch);
+#pragma unroll
+              for (int k = 0; k < kRowsPerWarp; ++k) {
+                const float4 qv = *reinterpret_cast<const float4 *>(q0 + k * D + ch);
+                s[k][0] = fmaf(qv.x, k0.x, s[k][0]);
+                s[k][0] = fmaf(qv.y, k0.y, s[k][0]);
+                s[k][0] = fmaf(qv.z, k0.z, s[k][0]);
+                s[k][0] = fmaf(qv.w, k0.w, s[k][0]);
+              }
+            }
+          } else
 #pragma unroll 2
           for (int ch = 0; ch < D; ch += 4) {
             const float4 k0 = *reinterpret_cast<const float4 *>(sK + lane * (D + 4) + ch);
