@@ -487,3 +487,103 @@ def values_f64(arr: np.ndarray, dtype: str) -> np.ndarray:
     if dtype == "bf16":
         return bf16_bits_to_f32(arr).astype(np.float64)
     return np.asarray(arr, np.float32).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# multi-turn timelines (Algorithm 1's outer loop)
+
+_T_TIMELINE = 32  # stream tags of the timeline draws (disjoint from the tags above)
+
+
+@dataclass
+class Timeline:
+    """A multi-turn agent trajectory q, z_1, a_1, o_1, ..., z_T, a_T, o_T,
+    z_{T+1} with one commit per tool call a_t.
+
+    events[j] = (kind, first token, length) in timeline order; commit t
+    (0-based) ends at commit_end[t] (the end of a_t); its pre-commit window
+    is the last W positions before commit_end[t] and its post-commit window
+    the first W tokens of the next reasoning event, which start at
+    post_start[t] (after the observation o_t).  Positions are the timeline
+    indices.  K, V [M][H][S][d], Q_pre / Q_post [T][M][Hq][W][d] (bf16 bits
+    or float32), fill [S] (a per-token score for the budget's fill)."""
+    cfg: Config
+    seed: int
+    turns: int
+    events: list
+    commit_end: np.ndarray
+    post_start: np.ndarray
+    K: np.ndarray = None
+    V: np.ndarray = None
+    Q_pre: np.ndarray = None
+    Q_post: np.ndarray = None
+    fill: np.ndarray = None
+
+    @property
+    def S(self):
+        kind, b, n = self.events[-1]
+        return b + n
+
+    def qpos_pre(self, t):
+        return np.arange(self.commit_end[t] - self.cfg.W, self.commit_end[t], dtype=np.int32)
+
+    def qpos_post(self, t):
+        return np.arange(self.post_start[t], self.post_start[t] + self.cfg.W, dtype=np.int32)
+
+
+def make_timeline(cfg: Config, seed: int = 0, turns: int = 3, values: bool = True) -> Timeline:
+    """Event lengths uniform in cfg.event_len (reasoning events at least W
+    long, so that a post-commit window lies inside the next reasoning event);
+    Q, K, V ~ N(0, 1) from the counter-based generator; fill uniform."""
+    dr = Draws(seed, _stream(0, _T_TIMELINE))
+    lo, hi = cfg.event_len
+    ev, t = [], 0
+
+    def add(kind, n):
+        nonlocal t
+        ev.append((kind, t, n))
+        t += n
+
+    add("query", dr.randint(lo, hi))
+    commit_end, post_start = [], []
+    for k in range(turns):
+        add("reason", dr.randint(max(lo, cfg.W), max(hi, cfg.W)))
+        add("call", dr.randint(lo, hi))
+        commit_end.append(t)
+        add("obs", dr.randint(lo, hi))
+        post_start.append(t)
+    add("reason", dr.randint(max(lo, cfg.W), max(hi, cfg.W)))
+    tl = Timeline(cfg, seed, turns, ev, np.asarray(commit_end, np.int32), np.asarray(post_start, np.int32))
+    if values:
+        bf = cfg.dtype == "bf16"
+        S, M, H, Hq, W, d = tl.S, cfg.M, cfg.H, cfg.Hq, cfg.W, cfg.d
+        tl.K = normal(seed, _stream(0, _T_TIMELINE + 1), (M, H, S, d), bf16=bf)
+        tl.V = normal(seed, _stream(0, _T_TIMELINE + 2), (M, H, S, d), bf16=bf)
+        tl.Q_pre = normal(seed, _stream(0, _T_TIMELINE + 3), (turns, M, Hq, W, d), bf16=bf)
+        tl.Q_post = normal(seed, _stream(0, _T_TIMELINE + 4), (turns, M, Hq, W, d), bf16=bf)
+        tl.fill = uniform_array(seed, _stream(0, _T_TIMELINE + 5), S)
+    return tl
+
+
+def timeline_steps(tl: Timeline):
+    """The order in which a timeline is fed to a lifecycle session:
+    ("append", a, b) the tokens [a, b); ("pre", t) commit t's pre-commit
+    measurement; ("checkpoint",) a compression checkpoint (taken when the
+    resident tokens exceed the budget); ("post", t) commit t's post-commit
+    measurement and decisions."""
+    steps, t0 = [], 0
+    for k in range(tl.turns):
+        steps.append(("append", t0, int(tl.commit_end[k])))
+        t0 = int(tl.commit_end[k])
+        steps.append(("pre", k))
+        steps.append(("checkpoint",))
+        end = int(tl.post_start[k]) + tl.cfg.W
+        steps.append(("append", t0, end))
+        t0 = end
+        steps.append(("post", k))
+    return steps
+
+
+def timeline_events(tl: Timeline, a: int, b: int):
+    """The paged events (tool calls, observations) that lie in [a, b)."""
+    return [(k, s, n) for k, s, n in tl.events if k in ("call", "obs") and a <= s and s + n <= b]
