@@ -506,7 +506,8 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
   static thread_local JointLaunch L;
   memset(&L, 0, sizeof L);
   fill_batch(L.batch, shape, n_traj, post, layer_mask);
-  int nl = L.batch.n_layers, g = L.batch.g, d = shape->head_dim, RB = joint_rows_per_group();
+  for (int t = 0; t < n_traj; ++t) L.stats[t] = stats[t];
+  int nl = L.batch.n_layers, g = L.batch.g, d = shape->head_dim, RB = joint_rows_per_group(L);
   size_t rows_total = 0;
   int maxP = 0;
   for (int t = 0; t < n_traj; ++t) {
@@ -532,7 +533,6 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
   L.roundR = reinterpret_cast<float *>(base);
   L.rows_full = (int64_t)rows_full;
   for (int t = 0; t < n_traj; ++t) {
-    L.stats[t] = stats[t];
     L.cand[t] = cand[t];
     L.accepted[t] = accepted_out[t];
     L.stepR_out[t] = step_R_out ? step_R_out[t] : nullptr;

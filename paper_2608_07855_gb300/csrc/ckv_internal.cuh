@@ -151,8 +151,13 @@ struct JointLaunch {
   int32_t row_off[kMaxTraj + 1];
   float tau;
 };
+// Tensor-core kernel (bf16, head_dim 128, 16-byte aligned rows) when the
+// launch allows it, else the CUDA-core kernel; the row-group size follows.
 cudaError_t launch_joint(const JointLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count);
-int joint_rows_per_group();
+int joint_rows_per_group(const JointLaunch &L);
+bool joint_tc_eligible(const JointLaunch &L);
+int joint_tc_rows_per_group();
+cudaError_t launch_joint_tc(const JointLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count);
 int joint_round();   // candidates per round
 int joint_combos();  // (candidate, earlier subset) pairs per round
 

@@ -21,73 +21,22 @@
 // The decisions and step values are those of the scan that takes one
 // candidate per barrier; deletion sums over disjoint pages add, which is what
 // Eq. 11's joint deletion needs.
-#include <cooperative_groups.h>
-
-#include "ckv_internal.cuh"
+#include "joint_common.cuh"
 #include "commitkv_testing.h"
 
 namespace ckv {
 namespace {
+
+using joint::combo;
+using joint::kCombos;
+using joint::kRound;
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kRowsPerWarp = 2;
 constexpr int kRB = kWarps * kRowsPerWarp;  // rows per group
 constexpr int kTK = 64;                     // page tokens per shared-memory chunk
-constexpr int kRound = 4;                   // candidates per round
-constexpr int kCombos = (1 << kRound) - 1;  // (candidate, subset of the earlier ones) pairs
 constexpr float kNegInf = -__builtin_huge_valf();
-constexpr uint64_t kWaitNs = 1000000000ull;  // 1 s per barrier
-
-static_assert(kRound * 4 <= 32, "accepted masks travel in one word");
-
-// Table slot of candidate c with the subset s of candidates 0..c-1.
-__host__ __device__ constexpr int combo(int c, int s) { return (1 << c) - 1 + s; }
-
-__device__ __forceinline__ int find_group_traj(const int32_t *off, int n, int unit) {
-  int t = 0;
-  while (t + 1 < n && unit >= off[t + 1]) ++t;
-  return t;
-}
-
-// Sense-free generation barrier over all blocks of a cooperative launch,
-// with a bounded wait.  Returns false (and records a timeout) on expiry.
-__device__ bool grid_barrier(WsHeader *hdr, unsigned nblocks) {
-  __shared__ int s_ok;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    volatile uint32_t *gen = &hdr->bar_gen;
-    volatile int32_t *abort_flag = &hdr->abort;
-    uint32_t g = *gen;
-    __threadfence();
-    uint32_t arrived = atomicAdd(&hdr->bar_count, 1u);
-    if (arrived == nblocks - 1) {
-      atomicExch(&hdr->bar_count, 0u);
-      __threadfence();
-      atomicAdd(&hdr->bar_gen, 1u);
-    } else {
-      uint64_t t0 = globaltimer_ns();
-      while (*gen == g) {
-        if (*abort_flag) {
-          ok = 0;
-          break;
-        }
-        if (globaltimer_ns() - t0 > kWaitNs) {
-          ok = 0;
-          atomicExch(&hdr->abort, 1);
-          record_error(hdr, COMMITKV_ERR_TIMEOUT, -3);
-          break;
-        }
-        __nanosleep(64);
-      }
-    }
-    __threadfence();
-    s_ok = ok;
-  }
-  __syncthreads();
-  return s_ok != 0;
-}
 
 // J consecutive floats (J = 2 or 4) as one vector access.
 template <int J>
@@ -128,7 +77,7 @@ struct Group {
 __device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
   const Batch &b = L.batch;
   Group G;
-  G.t = find_group_traj(L.group_off, b.n_traj, grp);
+  G.t = joint::find_group_traj(L.group_off, b.n_traj, grp);
   int local = grp - L.group_off[G.t], nrb = L.nrb[G.t];
   int rb = local % nrb;
   local /= nrb;
@@ -138,22 +87,6 @@ __device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
   G.rows = b.g * b.t[G.t].W;
   G.row0 = rb * kRB;
   return G;
-}
-
-// Candidates of round r for trajectory t (0 when the scan is over).
-__device__ __forceinline__ int round_count(const JointLaunch &L, int t, int r) {
-  int nc = min(max(L.n_cand[t], 0), L.batch.t[t].P);
-  return max(0, min(kRound, nc - r * kRound));
-}
-
-// The round's decisions, replayed from its table: bit c set = accepted.
-__device__ __forceinline__ unsigned resolve_round(const float *tab, int kc, float tau) {
-  unsigned acc = 0;
-  for (int c = 0; c < kc; ++c) {
-    float R = *(volatile const float *)(tab + combo(c, acc));
-    if (R <= tau) acc |= 1u << c;
-  }
-  return acc;
 }
 
 template <typename T, int D>
@@ -174,19 +107,15 @@ __global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constan
   const int ngroups = L.group_off[b.n_traj];
   const int64_t rows_full = L.rows_full;
 
-  int rounds = 0;
-  for (int t = 0; t < b.n_traj; ++t) {
-    int nc = min(max(L.n_cand[t], 0), b.t[t].P);
-    rounds = max(rounds, (nc + kRound - 1) / kRound);
-  }
+  const int rounds = joint::round_total(L);
 
   for (int r = 0; r < rounds; ++r) {
-    float *tab_r = L.roundR + (size_t)(r % 3) * b.n_traj * kCombos;
+    float *tab_r = joint::round_table(L, r);
     // ---------------- phase 1: the round's candidates on this block's rows
     for (int grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
       const Group G = decode_group(L, grp);
       const TrajDev &tr = b.t[G.t];
-      const int kc = round_count(L, G.t, r);
+      const int kc = joint::round_count(L, G.t, r);
       if (kc == 0) continue;
       __syncthreads();
       for (int e = threadIdx.x; e < kRB * D; e += kThreads) {
@@ -403,13 +332,13 @@ __global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constan
         atomic_max_nonneg(tab_r + G.t * kCombos + threadIdx.x, s_rmax[threadIdx.x]);
     }
     // ---------------- barrier: every block's part of the round's table is in
-    if (!grid_barrier(hdr, gridDim.x)) return;
+    if (!joint::grid_barrier(hdr, gridDim.x)) return;
     // ---------------- phase 2: replay the decisions, add the accepted sums
     for (int grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
       const Group G = decode_group(L, grp);
-      const int kc = round_count(L, G.t, r);
+      const int kc = joint::round_count(L, G.t, r);
       if (kc == 0) continue;
-      const unsigned acc = resolve_round(tab_r + G.t * kCombos, kc, L.tau);
+      const unsigned acc = joint::resolve_round(tab_r + G.t * kCombos, kc, L.tau);
       if (acc == 0) continue;
 #pragma unroll 1
       for (int k = 0; k < kRowsPerWarp; ++k) {
@@ -433,27 +362,7 @@ __global__ void __launch_bounds__(kThreads, 2) joint_kernel(const __grid_constan
         }
       }
     }
-    if (blockIdx.x == 0) {
-      for (int t = threadIdx.x; t < b.n_traj; t += kThreads) {
-        const int kc = round_count(L, t, r);
-        float *tab = tab_r + t * kCombos;
-        unsigned acc = 0;
-        for (int c = 0; c < kc; ++c) {
-          const int j = r * kRound + c;
-          const int E = L.cand[t][j];
-          const float R = *(volatile float *)(tab + combo(c, acc));
-          if (L.stepR_out[t]) L.stepR_out[t][j] = R;
-          if (R <= L.tau) {
-            acc |= 1u << c;
-            if (E >= 0 && E < b.t[t].P) L.accepted[t][E] = 1;
-          }
-        }
-        // the table of round r + 2 starts from zero (the last reads of this
-        // slot were in phase 2 of round r - 1, before this round's barrier)
-        float *next = L.roundR + (size_t)((r + 2) % 3) * b.n_traj * kCombos + t * kCombos;
-        for (int i = 0; i < kCombos; ++i) next[i] = 0.0f;
-      }
-    }
+    if (blockIdx.x == 0) joint::publish_round(L, r);
   }
 }
 
@@ -479,6 +388,7 @@ cudaError_t launch_joint_typed(const JointLaunch &L, WsHeader *hdr, cudaStream_t
 }  // namespace
 
 cudaError_t launch_joint(const JointLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count) {
+  if (joint_tc_eligible(L)) return launch_joint_tc(L, hdr, stream, sm_count);
   bool bf = L.batch.dtype == COMMITKV_BF16;
   if (L.batch.d == 128)
     return bf ? launch_joint_typed<__nv_bfloat16, 128>(L, hdr, stream, sm_count)
@@ -487,12 +397,12 @@ cudaError_t launch_joint(const JointLaunch &L, WsHeader *hdr, cudaStream_t strea
             : launch_joint_typed<float, 64>(L, hdr, stream, sm_count);
 }
 
-int joint_rows_per_group() { return kRB; }
+int joint_rows_per_group(const JointLaunch &L) { return joint_tc_eligible(L) ? joint_tc_rows_per_group() : kRB; }
 int joint_round() { return kRound; }
 int joint_combos() { return kCombos; }
 
 namespace {
-__global__ void barrier_timeout_kernel(WsHeader *hdr, unsigned expected) { grid_barrier(hdr, expected); }
+__global__ void barrier_timeout_kernel(WsHeader *hdr, unsigned expected) { joint::grid_barrier(hdr, expected); }
 }  // namespace
 
 }  // namespace ckv

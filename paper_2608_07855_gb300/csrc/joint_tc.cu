@@ -1,0 +1,521 @@
+// Greedy joint test (Section 3.4, Eq. 11) on the 5th-generation tensor
+// cores: bf16 K/V/Q, head_dim 128, fp32 accumulation in tensor memory.
+//
+// One cooperative persistent kernel, one CTA of 128 threads per SM.  A
+// group is 128 probe rows of one (trajectory, selected layer, KV head):
+// thread i and TMEM lane i hold row i.  In every round (joint_common.cuh) a
+// group makes up to two passes of the same machinery over a list of at
+// most four pages:
+//   fold  the pages of the previous round that were accepted: their D_E are
+//         computed again (bit-identical to the values that round used) and
+//         added, in candidate order, into the row's D_A, S_A, n_A in the
+//         workspace;
+//   scan  the round's candidates: Eq. 6 on A u T for every non-empty subset
+//         T of them, max over the rows (Eq. 7) into the round's table.
+// A pass stages Q (once per group and round) and the pages' K and V rows in
+// shared memory (cp.async into the 128-byte-swizzled layout) and issues
+//   S = Q K^T       one MMA chain with N = 64 x pages, TMEM columns 256..511
+//   e = exp(s - m)  per row on the page's visible tokens (m = the row's
+//                   final max); S_E = sum e, n_E = count; P = e written
+//                   over S as a bf16 (hi, lo) pair
+//   U_E = P V_E     per page and 64-channel half, TMEM columns 64 c, TS form
+//                   (P from tensor memory, V from shared memory)
+// and the epilogue reads U_E 16 columns at a time: D_E = U_E - S_E o.  In
+// the scan the sums of the subsets are built as a tree in which every
+// subset adds its largest page last, so each is the sum that the
+// one-page-at-a-time scan forms, ((D_A + D_b1) + D_b2) + ... + D_c, and its
+// squared norm accumulates over the channels in order.
+// Pages longer than 64 tokens are taken in 64-token chunks: U accumulates
+// over the chunks, and the chunks' QK and softmax are redone for the second
+// channel half.  Every mbarrier wait is bounded (1 s); on expiry the kernel
+// records COMMITKV_ERR_TIMEOUT, raises the abort flag that the grid barrier
+// watches, waits (bounded) for its MMAs in flight, frees its tensor memory
+// and returns.
+#include "joint_common.cuh"
+#include "sm103.cuh"
+
+namespace ckv {
+namespace {
+
+using namespace ckv::sm103;
+using joint::kCombos;
+using joint::kRound;
+
+constexpr int D = 128;
+constexpr int kRows = 128;   // probe rows per group (MMA M, TMEM lanes)
+constexpr int kCT = 64;      // page tokens per chunk (the QK N of one page)
+constexpr int kThreads = 128;
+constexpr uint64_t kWait = 1000000000ull;
+constexpr uint32_t kQHalf = kRows * 128;         // one 64-channel half of the Q tile: 16 KB
+constexpr uint32_t kKHalf = kRound * kCT * 128;  // K rows of all pages, one half: 32 KB
+constexpr uint32_t kVHalf = kCT * 128;           // V rows of one page, one half: 8 KB
+constexpr uint32_t kColS = 256;                  // TMEM column of page 0's S/P (64 per page)
+
+struct SmemJ {
+  alignas(1024) uint8_t q[2 * kQHalf];
+  alignas(1024) uint8_t k[2 * kKHalf];
+  alignas(1024) uint8_t v[kRound][2 * kVHalf];
+  int pos[kRound][kCT];
+  unsigned rmax[16];
+  uint64_t bar;
+  uint32_t tmem;
+  int abort_flag;
+};
+
+struct Group {
+  int t, l, li, kvh, rows, row0;
+};
+
+// What a thread keeps of its probe row.
+struct Row {
+  bool ok;          // inside the group
+  int64_t grow;     // index into D_A, S_A
+  const float *st;  // stats row: m, l, n, pad, o[D]
+  float m2, l;      // final max in base-2 units, exp-sum
+  int nvis, qp;
+  float SA;
+  int nA;
+};
+
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// K-major tile of 128-byte rows in two 64-channel halves half_bytes apart:
+// the descriptor of k-step ks (16 channels).
+__device__ __forceinline__ uint64_t desc_kmajor(const uint8_t *tile, uint32_t half_bytes, int ks) {
+  return smem_desc(smem_addr(tile) + (ks >> 2) * half_bytes + (ks & 3) * 32, 16, 1024, kSwizzle128B);
+}
+// V rows of one page as the MN-major B operand (k = tokens, n = the 64
+// channels of half h): k-step ks (16 tokens).
+__device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int h, int ks) {
+  return smem_desc(smem_addr(tile) + h * kVHalf + ks * 2048, kVHalf, 1024, kSwizzle128B);
+}
+// TMEM column of the 8 packed P columns (hi or lo) of page c, k-step ks.
+__device__ __forceinline__ uint32_t p_col(int c, int ks, int lo) {
+  return kColS + 64 * c + 32 * (ks >> 1) + 8 * (ks & 1) + 16 * lo;
+}
+
+__device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
+  const Batch &b = L.batch;
+  Group G;
+  G.t = joint::find_group_traj(L.group_off, b.n_traj, grp);
+  int local = grp - L.group_off[G.t], nrb = L.nrb[G.t];
+  const int rb = local % nrb;
+  local /= nrb;
+  G.kvh = local % b.H;
+  G.li = local / b.H;
+  G.l = b.layer_ids[G.li];
+  G.rows = b.g * b.t[G.t].W;
+  G.row0 = rb * kRows;
+  return G;
+}
+
+// Waits for the MMAs committed to the pass barrier; uniform over the block.
+__device__ __forceinline__ bool wait_mma(SmemJ &s, uint32_t &phase) {
+  bool ok = mbar_wait(&s.bar, phase, kWait, &s.abort_flag);
+  phase ^= 1u;
+  ok = __syncthreads_and(ok) != 0;
+  if (ok) tc_fence_after();
+  return ok;
+}
+
+// o and D_A of kSub channels of the thread's row.
+constexpr int kSub = 8;
+__device__ __forceinline__ void load_sub(const Row &rw, const float *DA, int ch0, float (&o)[kSub],
+                                         float (&da)[kSub]) {
+  if (rw.ok) {
+    const float4 *po = reinterpret_cast<const float4 *>(rw.st + 4 + ch0);
+    const float4 *pa = reinterpret_cast<const float4 *>(DA + rw.grow * D + ch0);
+#pragma unroll
+    for (int u = 0; u < kSub / 4; ++u) {
+      const float4 x = po[u], y = pa[u];
+      o[4 * u] = x.x, o[4 * u + 1] = x.y, o[4 * u + 2] = x.z, o[4 * u + 3] = x.w;
+      da[4 * u] = y.x, da[4 * u + 1] = y.y, da[4 * u + 2] = y.z, da[4 * u + 3] = y.w;
+    }
+  } else {
+#pragma unroll
+    for (int u = 0; u < kSub; ++u) o[u] = da[u] = 0.0f;
+  }
+}
+
+// 32 lanes x 8 consecutive 32-bit columns.
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[kSub]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+               : "r"(taddr));
+}
+
+// Largest member of the non-empty set T (a constant after unrolling).
+__host__ __device__ constexpr int top_bit(int T) { return T >= 8 ? 3 : T >= 4 ? 2 : T >= 2 ? 1 : 0; }
+
+// One pass over the pages list[0..n) (n <= kRound).  kScan: accumulates the
+// squared norms of the subset sums into ss and o's squared norm into on2;
+// otherwise adds the pages' D_E into D_A in the workspace.  S_E and n_E of
+// each page are left in Sc and nc.  Returns false on a timeout.
+template <bool kScan>
+__device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeader *hdr, const Group &G,
+                                         const Row &rw, const int *list, int n, bool stage_q, uint32_t tm,
+                                         uint32_t lane_base, uint32_t &phase, float (&ss)[kCombos], float &on2,
+                                         float (&Sc)[kRound], int (&nc)[kRound]) {
+  const Batch &b = L.batch;
+  const TrajDev &tr = b.t[G.t];
+  const int tid = threadIdx.x;
+  int ps[kRound], pl[kRound];
+  int nch = 1;
+#pragma unroll
+  for (int c = 0; c < kRound; ++c) {
+    ps[c] = pl[c] = 0;
+    Sc[c] = 0.0f;
+    nc[c] = 0;
+    if (c < n) {
+      const int E = list[c];
+      if (E < 0 || E >= tr.P) {
+        if (tid == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, -4);
+      } else {
+        ps[c] = tr.ps[E];
+        pl[c] = tr.pl[E];
+        if (pl[c] < 0 || ps[c] < 0 || ps[c] > tr.S - pl[c]) {
+          if (tid == 0) record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, E);
+          ps[c] = pl[c] = 0;
+        }
+      }
+      nch = max(nch, (pl[c] + kCT - 1) / kCT);
+    }
+  }
+  const __nv_bfloat16 *kp =
+      static_cast<const __nv_bfloat16 *>(tr.k) + (int64_t)G.l * tr.sl + (int64_t)G.kvh * tr.sh;
+  const __nv_bfloat16 *vp =
+      static_cast<const __nv_bfloat16 *>(tr.v) + (int64_t)G.l * tr.sl + (int64_t)G.kvh * tr.sh;
+
+  for (int h = 0; h < 2; ++h) {
+    for (int j = 0; j < nch; ++j) {
+      int nt[kRound];
+#pragma unroll
+      for (int c = 0; c < kRound; ++c) nt[c] = c < n ? min(kCT, max(0, pl[c] - j * kCT)) : 0;
+      if (h == 0 || nch > 1) {
+        // ---- stage (the MMAs that read the buffers have completed)
+        __syncthreads();
+        if (stage_q && h == 0 && j == 0) {
+          for (int e = tid; e < kRows * 16; e += kThreads) {
+            const int r = e >> 4, k16 = e & 15, row = G.row0 + r;
+            if (row < G.rows) {
+              const int hq = G.kvh * b.g + row / tr.W, w = row % tr.W;
+              const __nv_bfloat16 *src =
+                  static_cast<const __nv_bfloat16 *>(tr.q) + (((int64_t)G.l * b.Hq + hq) * tr.W + w) * D + 8 * k16;
+              cp_async16(s.q + (k16 >> 3) * kQHalf + sw128_offset(r, k16 & 7), src);
+            }
+          }
+        }
+        for (int e = tid; e < n * kCT * 16; e += kThreads) {
+          const int c = e / (kCT * 16), rem = e % (kCT * 16), i = rem >> 4, k16 = rem & 15;
+          if (i < nt[c]) {
+            const int64_t off = (int64_t)(ps[c] + j * kCT + i) * tr.st + 8 * k16;
+            cp_async16(s.k + (k16 >> 3) * kKHalf + sw128_offset(kCT * c + i, k16 & 7), kp + off);
+            cp_async16(s.v[c] + (k16 >> 3) * kVHalf + sw128_offset(i, k16 & 7), vp + off);
+          }
+        }
+        for (int e = tid; e < n * kCT; e += kThreads) {
+          const int c = e / kCT, i = e % kCT;
+          s.pos[c][i] = i < nt[c] ? tr.pos[ps[c] + j * kCT + i] : 0;
+        }
+        cp_async_wait_all();
+        fence_proxy_async();
+        __syncthreads();
+        // ---- S = Q K^T for all pages of the pass
+        if (tid == 0) {
+          tc_fence_after();
+          const uint32_t idesc = idesc_bf16_f32(kRows, kCT * n, 0, 0);
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks)
+            mma_bf16(tm + kColS, desc_kmajor(s.q, kQHalf, ks), desc_kmajor(s.k, kKHalf, ks), idesc, ks > 0);
+          mma_commit(&s.bar);
+        }
+        if (!wait_mma(s, phase)) return false;
+        // ---- e = exp(s - m) on the visible tokens; P over S
+#pragma unroll 1
+        for (int c = 0; c < n; ++c) {
+          const int nblk = max(1, (nt[c] + 31) / 32);
+#pragma unroll 1
+          for (int jb = 0; jb < nblk; ++jb) {
+            float x[32];
+            uint32_t pk[32];
+            const uint32_t addr = tm + lane_base + kColS + 64 * c + 32 * jb;
+            tmem_ld32f(addr, x);
+            tmem_wait_ld();
+            float se = 0.0f;
+            int ne = 0;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int tok = 32 * jb + i;
+              const bool vis = rw.ok && tok < nt[c] && s.pos[c][tok] <= rw.qp;
+              const float e = vis ? exp2f(x[i] * b.scale_log2 - rw.m2) : 0.0f;
+              se += e;
+              ne += vis ? 1 : 0;
+              x[i] = e;
+            }
+            if (h == 0) {
+              Sc[c] += se;
+              nc[c] += ne;
+            }
+            split_pack32(x, pk);
+            tmem_st32(addr, pk);
+          }
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+      }
+      // ---- U_E (+)= P V_E for channel half h
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t idesc = idesc_bf16_f32(kRows, 64, 0, 1);
+#pragma unroll 1
+        for (int c = 0; c < n; ++c) {
+          const int nks = max(1, (nt[c] + 15) / 16);
+#pragma unroll 1
+          for (int ks = 0; ks < nks; ++ks) {
+            const uint64_t bd = desc_v(s.v[c], h, ks);
+            mma_bf16_ts(tm + 64 * c, tm + p_col(c, ks, 0), bd, idesc, (j > 0 || ks > 0) ? 1u : 0u);
+            mma_bf16_ts(tm + 64 * c, tm + p_col(c, ks, 1), bd, idesc, 1u);
+          }
+        }
+        mma_commit(&s.bar);
+      }
+      const bool last = j == nch - 1;
+      float o[kSub], da[kSub];
+      if (last) load_sub(rw, L.DA, 64 * h, o, da);  // in flight while the MMAs run
+      if (!wait_mma(s, phase)) return false;
+      if (last) {
+        // ---- epilogue over the 64 channels of half h, kSub at a time
+#pragma unroll 1
+        for (int q = 0; q < 64 / kSub; ++q) {
+          const int ch0 = 64 * h + kSub * q;
+          float o_n[kSub], da_n[kSub];
+          if (q + 1 < 64 / kSub) load_sub(rw, L.DA, ch0 + kSub, o_n, da_n);
+          uint32_t u[kRound][kSub];
+#pragma unroll
+          for (int c = 0; c < kRound; ++c)
+            if (c < n) tmem_ld8(tm + lane_base + 64 * c + kSub * q, u[c]);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < kSub; ++i) {
+            float de[kRound];
+#pragma unroll
+            for (int c = 0; c < kRound; ++c) de[c] = c < n ? fmaf(-Sc[c], o[i], __uint_as_float(u[c][i])) : 0.0f;
+            if constexpr (kScan) {
+              on2 = fmaf(o[i], o[i], on2);
+              float p[1 << kRound];
+              p[0] = da[i];
+#pragma unroll
+              for (int T = 1; T < (1 << kRound); ++T) {
+                p[T] = p[T & ~(1 << top_bit(T))] + de[top_bit(T)];
+                ss[T - 1] = fmaf(p[T], p[T], ss[T - 1]);
+              }
+            } else {
+              float x = da[i];
+#pragma unroll
+              for (int c = 0; c < kRound; ++c)
+                if (c < n) x += de[c];
+              da[i] = x;
+            }
+          }
+          if constexpr (!kScan) {
+            if (rw.ok) {
+              float4 *pa = reinterpret_cast<float4 *>(L.DA + rw.grow * D + ch0);
+#pragma unroll
+              for (int u4 = 0; u4 < kSub / 4; ++u4)
+                pa[u4] = make_float4(da[4 * u4], da[4 * u4 + 1], da[4 * u4 + 2], da[4 * u4 + 3]);
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < kSub; ++i) {
+            o[i] = o_n[i];
+            da[i] = da_n[i];
+          }
+        }
+      }
+      // the epilogue's TMEM reads are done before the next MMAs write
+      tc_fence_before();
+      __syncthreads();
+    }
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_constant__ JointLaunch L,
+                                                             WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  SmemJ &s = *reinterpret_cast<SmemJ *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const Batch &b = L.batch;
+  const int tid = threadIdx.x, warp = tid / 32, lane = tid % 32;
+
+  // Rows past a page's end are never written: they keep finite values (zero
+  // or an earlier page's), whose scores are masked and whose V rows meet
+  // P = 0.
+  for (int i = tid; i < (int)(sizeof(s.q) / 16); i += kThreads) reinterpret_cast<uint4 *>(s.q)[i] = uint4{};
+  for (int i = tid; i < (int)(sizeof(s.k) / 16); i += kThreads) reinterpret_cast<uint4 *>(s.k)[i] = uint4{};
+  for (int i = tid; i < (int)(sizeof(s.v) / 16); i += kThreads) reinterpret_cast<uint4 *>(&s.v[0][0])[i] = uint4{};
+  if (tid == 0) {
+    s.abort_flag = 0;
+    mbar_init(&s.bar, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&s.tmem, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = s.tmem;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  uint32_t phase = 0;
+  bool ok = true;
+
+  const int rounds = joint::round_total(L);
+  const int ngroups = L.group_off[b.n_traj];
+  for (int r = 0; r < rounds && ok; ++r) {
+    float *tab_r = joint::round_table(L, r);
+    for (int grp = blockIdx.x; grp < ngroups; grp += gridDim.x) {
+      const Group G = decode_group(L, grp);
+      const TrajDev &tr = b.t[G.t];
+      const int kc = joint::round_count(L, G.t, r);
+      if (kc == 0) continue;
+      // the previous round's accepted pages, in candidate order
+      int fold[kRound], nf = 0;
+      if (r > 0) {
+        const int kp = joint::round_count(L, G.t, r - 1);
+        const unsigned acc =
+            joint::resolve_round(joint::round_table(L, r - 1) + G.t * kCombos, kp, L.tau);
+        for (int c = 0; c < kp; ++c)
+          if ((acc >> c) & 1u) fold[nf++] = L.cand[G.t][(r - 1) * kRound + c];
+      }
+      int cand[kRound];
+      for (int c = 0; c < kc; ++c) cand[c] = L.cand[G.t][r * kRound + c];
+
+      Row rw;
+      const int row = G.row0 + tid;
+      rw.ok = row < G.rows;
+      const int hq = G.kvh * b.g + (rw.ok ? row / tr.W : 0), w = rw.ok ? row % tr.W : 0;
+      rw.grow = L.row_off[G.t] + (int64_t)(G.li * b.H + G.kvh) * G.rows + (rw.ok ? row : 0);
+      rw.st = L.stats[G.t] + (((int64_t)G.l * b.Hq + hq) * tr.W + w) * (D + 4);
+      const float mn = rw.ok ? rw.st[0] : -__builtin_huge_valf();
+      rw.m2 = mn == -__builtin_huge_valf() ? mn : mn * 1.4426950408889634f;
+      rw.l = rw.ok ? rw.st[1] : 0.0f;
+      rw.nvis = rw.ok ? (int)rw.st[2] : 0;
+      rw.qp = rw.ok ? tr.qpos[w] : -0x7fffffff;
+      rw.SA = rw.ok ? L.SA[rw.grow * 2] : 0.0f;
+      rw.nA = rw.ok ? (int)L.SA[rw.grow * 2 + 1] : 0;
+      if (tid < 16) s.rmax[tid] = 0u;
+
+      float ss[kCombos], on2 = 0.0f, Sc[kRound];
+      int nc[kRound];
+#pragma unroll
+      for (int i = 0; i < kCombos; ++i) ss[i] = 0.0f;
+      if (nf > 0) {
+        if (!run_pass<false>(s, L, hdr, G, rw, fold, nf, true, tm, lane_base, phase, ss, on2, Sc, nc)) {
+          ok = false;
+          break;
+        }
+#pragma unroll
+        for (int c = 0; c < kRound; ++c)
+          if (c < nf) {
+            rw.SA += Sc[c];
+            rw.nA += nc[c];
+          }
+        if (rw.ok) {
+          L.SA[rw.grow * 2] = rw.SA;
+          L.SA[rw.grow * 2 + 1] = (float)rw.nA;
+        }
+      }
+      if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, ss, on2, Sc, nc)) {
+        ok = false;
+        break;
+      }
+      // Eq. 6 on A u T for every non-empty subset T of the round's pages;
+      // S and n added in candidate order
+      const float onorm = sqrtf(on2);
+#pragma unroll
+      for (int T = 1; T < (1 << kRound); ++T) {
+        if (T >= (1 << kc)) break;
+        float S_tot = rw.SA;
+        int n_tot = rw.nA;
+#pragma unroll
+        for (int c = 0; c < kRound; ++c)
+          if ((T >> c) & 1) {
+            S_tot += Sc[c];
+            n_tot += nc[c];
+          }
+        const float rv = rw.ok ? effect_value(n_tot, rw.nvis, S_tot, rw.l, ss[T - 1], onorm) : 0.0f;
+        const unsigned mx = __reduce_max_sync(0xffffffffu, __float_as_uint(rv));
+        if (lane == 0) atomicMax(&s.rmax[T - 1], mx);
+      }
+      __syncthreads();
+      if (tid < (1 << kc) - 1) atomic_max_nonneg(tab_r + G.t * kCombos + tid, __uint_as_float(s.rmax[tid]));
+    }
+    if (!ok) break;
+    if (!joint::grid_barrier(hdr, gridDim.x)) {
+      ok = false;
+      break;
+    }
+    if (blockIdx.x == 0) joint::publish_round(L, r);
+  }
+
+  if (!ok) {
+    // a wait ran out (or another block gave up): leave the grid barrier to
+    // the others and let the MMAs in flight finish before the memory goes
+    if (tid == 0) {
+      if (s.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, -5);
+      atomicExch(&hdr->abort, 1);
+      mbar_wait_drain(&s.bar, phase ^ 1u, kWait);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
+}
+
+}  // namespace
+
+// bf16, head_dim 128, and 16-byte aligned rows of K, V, Q and the stats.
+bool joint_tc_eligible(const JointLaunch &L) {
+  const Batch &b = L.batch;
+  if (b.dtype != COMMITKV_BF16 || b.d != D) return false;
+  for (int t = 0; t < b.n_traj; ++t) {
+    const TrajDev &tr = b.t[t];
+    if (tr.P == 0 || tr.W == 0) continue;
+    if ((reinterpret_cast<uintptr_t>(tr.k) | reinterpret_cast<uintptr_t>(tr.v) |
+         reinterpret_cast<uintptr_t>(tr.q) | reinterpret_cast<uintptr_t>(L.stats[t])) & 15)
+      return false;
+    if ((tr.sl | tr.sh | tr.st) & 7) return false;
+  }
+  return true;
+}
+
+int joint_tc_rows_per_group() { return kRows; }
+
+cudaError_t launch_joint_tc(const JointLaunch &L, WsHeader *hdr, cudaStream_t stream, int sm_count) {
+  const size_t smem = sizeof(SmemJ) + 1024;
+  cudaError_t e = cudaFuncSetAttribute(joint_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, joint_tc_kernel, kThreads, smem);
+  if (e != cudaSuccess) return e;
+  // one CTA per SM: each takes all 512 TMEM columns
+  if (per_sm != 1) return cudaErrorInvalidConfiguration;
+  const int ngroups = L.group_off[L.batch.n_traj];
+  const int grid = ngroups < sm_count ? ngroups : sm_count;
+  if (grid < 1) return cudaSuccess;
+  void *args[] = {(void *)&L, (void *)&hdr};
+  return cudaLaunchCooperativeKernel((const void *)joint_tc_kernel, dim3(grid), dim3(kThreads), args, smem,
+                                     stream);
+}
+
+}  // namespace ckv
