@@ -334,13 +334,13 @@ def buf_launches(buf):
     sequence of each call).  Scoring, one call over the 2n pre- and
     post-commit caches: on the tensor-core path (bf16, head_dim 128) prep +
     pass A + combine + pass B for every group of up to 16 caches, else pass A
-    + combine + pass B; classify 1; joint test 1; compaction = select +
-    gather."""
+    + combine + pass B; classify = per-page states + candidate order; joint
+    test 1; compaction = select + gather."""
     cfg = buf.cfg
     tc = cfg.dtype == "bf16" and cfg.d == 128 and os.environ.get("COMMITKV_SCORING") != "simt"
     n = 2 * len(buf.trajs)
     score = 4 * ((n + 15) // 16) if tc else 3
-    return score + 1 + 1 + 2
+    return score + 2 + 1 + 2
 
 
 def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):

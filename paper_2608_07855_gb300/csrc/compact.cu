@@ -62,7 +62,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
   __shared__ uint8_t s_take[kMaxPending];
   __shared__ unsigned s_hist[256];
   __shared__ unsigned long long s_prefix;
-  __shared__ int s_krem;
+  __shared__ int s_krem, s_exact;
 
   if (threadIdx.x == 0) {
     s_bad = 0;
@@ -160,8 +160,11 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
     if (threadIdx.x == 0) {
       s_prefix = 0ull;
       s_krem = room;
+      s_exact = 0;
     }
     unsigned long long mask = 0ull;
+    // stops early once every key with the chosen prefix is taken: the
+    // prefix (lower bits zero) is then itself the threshold
     for (int shift = 56; shift >= 0 && room > 0; shift -= 8) {
       for (int d = threadIdx.x; d < 256; d += kThreads) s_hist[d] = 0;
       __syncthreads();
@@ -179,6 +182,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
           if (cum + s_hist[d] >= (unsigned)need) {
             s_prefix = prefix | ((unsigned long long)d << shift);
             s_krem = need - (int)cum;
+            s_exact = s_krem == (int)s_hist[d];
             break;
           }
           cum += s_hist[d];
@@ -186,6 +190,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
       }
       mask |= 255ull << shift;
       __syncthreads();
+      if (s_exact) break;
     }
     unsigned long long thr = s_prefix;
     for (int i = threadIdx.x; i < S; i += kThreads)
@@ -195,17 +200,17 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
       if (cls[i] == 0) cls[i] = 3;
   }
   __syncthreads();
-  // I_j ascending: protected (2) and kept (3) tokens
-  int base = 0;
-  for (int c0 = 0; c0 < S; c0 += kThreads) {
-    int i = c0 + threadIdx.x;
-    int keep = i < S && cls[i] >= 2;
-    int excl;
-    int total = block_scan(keep, &excl, s_warp);
-    if (keep && base + excl < L.B) L.idx[t][base + excl] = i;
-    base += total;
-  }
-  if (threadIdx.x == 0) L.n_idx[t] = base < L.B ? base : L.B;
+  // I_j ascending: protected (2) and kept (3) tokens; each thread takes a
+  // contiguous segment, one block scan places the segments
+  const int seg = (S + kThreads - 1) / kThreads;
+  const int i0 = min(S, (int)threadIdx.x * seg), i1 = min(S, i0 + seg);
+  int cnt = 0;
+  for (int i = i0; i < i1; ++i) cnt += cls[i] >= 2;
+  int excl;
+  const int total = block_scan(cnt, &excl, s_warp);
+  for (int i = i0, o = excl; i < i1 && o < L.B; ++i)
+    if (cls[i] >= 2) L.idx[t][o++] = i;
+  if (threadIdx.x == 0) L.n_idx[t] = total < L.B ? total : L.B;
 }
 
 template <int VEC_BYTES>

@@ -43,18 +43,23 @@ using joint::kRound;
 
 constexpr int D = 128;
 constexpr int kRows = 128;   // probe rows per group (MMA M, TMEM lanes)
-constexpr int kCT = 64;      // page tokens per chunk (the QK N of one page)
+constexpr int kCT = 32;      // page tokens per chunk (the QK N of one page)
 constexpr int kThreads = 128;
 constexpr uint64_t kWait = 1000000000ull;
 constexpr uint32_t kQHalf = kRows * 128;         // one 64-channel half of the Q tile: 16 KB
-constexpr uint32_t kKHalf = kRound * kCT * 128;  // K rows of all pages, one half: 32 KB
-constexpr uint32_t kVHalf = kCT * 128;           // V rows of one page, one half: 8 KB
-constexpr uint32_t kColS = 256;                  // TMEM column of page 0's S/P (64 per page)
+constexpr uint32_t kKHalf = kRound * kCT * 128;  // K rows of all pages, one half: 16 KB
+constexpr uint32_t kVHalf = kCT * 128;           // V rows of one page, one half: 4 KB
+constexpr uint32_t kColS = 256;                  // TMEM column of page 0's S/P (kCT per page)
+constexpr int kHalfPad = 68;                     // floats per row of the o / D_A half buffers
 
 struct SmemJ {
   alignas(1024) uint8_t q[2 * kQHalf];
   alignas(1024) uint8_t k[2 * kKHalf];
   alignas(1024) uint8_t v[kRound][2 * kVHalf];
+  // o and D_A of one 64-channel half of every row (each thread its own
+  // row; the padding keeps the rows' 16-byte words in distinct banks)
+  alignas(16) float oh[kRows][kHalfPad];
+  alignas(16) float dah[kRows][kHalfPad];
   int pos[kRound][kCT];
   unsigned rmax[16];
   uint64_t bar;
@@ -96,8 +101,9 @@ __device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int h, int ks) {
 }
 // TMEM column of the 8 packed P columns (hi or lo) of page c, k-step ks.
 __device__ __forceinline__ uint32_t p_col(int c, int ks, int lo) {
-  return kColS + 64 * c + 32 * (ks >> 1) + 8 * (ks & 1) + 16 * lo;
+  return kColS + kCT * c + 32 * (ks >> 1) + 8 * (ks & 1) + 16 * lo;
 }
+static_assert(kCT == 32, "one 32-column TMEM load covers a page chunk's scores");
 
 __device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
   const Batch &b = L.batch;
@@ -123,22 +129,17 @@ __device__ __forceinline__ bool wait_mma(SmemJ &s, uint32_t &phase) {
   return ok;
 }
 
-// o and D_A of kSub channels of the thread's row.
-constexpr int kSub = 8;
-__device__ __forceinline__ void load_sub(const Row &rw, const float *DA, int ch0, float (&o)[kSub],
-                                         float (&da)[kSub]) {
-  if (rw.ok) {
-    const float4 *po = reinterpret_cast<const float4 *>(rw.st + 4 + ch0);
-    const float4 *pa = reinterpret_cast<const float4 *>(DA + rw.grow * D + ch0);
+constexpr int kSub = 8;  // channels per epilogue step
+
+// Starts the copies of o and D_A of channel half h of the thread's own row
+// into its rows of the half buffers.
+__device__ __forceinline__ void stage_half(SmemJ &s, const Row &rw, const float *DA, int h) {
+  if (!rw.ok) return;
+  const int i = threadIdx.x;
 #pragma unroll
-    for (int u = 0; u < kSub / 4; ++u) {
-      const float4 x = po[u], y = pa[u];
-      o[4 * u] = x.x, o[4 * u + 1] = x.y, o[4 * u + 2] = x.z, o[4 * u + 3] = x.w;
-      da[4 * u] = y.x, da[4 * u + 1] = y.y, da[4 * u + 2] = y.z, da[4 * u + 3] = y.w;
-    }
-  } else {
-#pragma unroll
-    for (int u = 0; u < kSub; ++u) o[u] = da[u] = 0.0f;
+  for (int u = 0; u < 16; ++u) {
+    cp_async16(&s.oh[i][4 * u], rw.st + 4 + 64 * h + 4 * u);
+    cp_async16(&s.dah[i][4 * u], DA + rw.grow * D + 64 * h + 4 * u);
   }
 }
 
@@ -238,32 +239,27 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
         // ---- e = exp(s - m) on the visible tokens; P over S
 #pragma unroll 1
         for (int c = 0; c < n; ++c) {
-          const int nblk = max(1, (nt[c] + 31) / 32);
-#pragma unroll 1
-          for (int jb = 0; jb < nblk; ++jb) {
-            float x[32];
-            uint32_t pk[32];
-            const uint32_t addr = tm + lane_base + kColS + 64 * c + 32 * jb;
-            tmem_ld32f(addr, x);
-            tmem_wait_ld();
-            float se = 0.0f;
-            int ne = 0;
+          float x[32];
+          uint32_t pk[32];
+          const uint32_t addr = tm + lane_base + kColS + kCT * c;
+          tmem_ld32f(addr, x);
+          tmem_wait_ld();
+          float se = 0.0f;
+          int ne = 0;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int tok = 32 * jb + i;
-              const bool vis = rw.ok && tok < nt[c] && s.pos[c][tok] <= rw.qp;
-              const float e = vis ? exp2f(x[i] * b.scale_log2 - rw.m2) : 0.0f;
-              se += e;
-              ne += vis ? 1 : 0;
-              x[i] = e;
-            }
-            if (h == 0) {
-              Sc[c] += se;
-              nc[c] += ne;
-            }
-            split_pack32(x, pk);
-            tmem_st32(addr, pk);
+          for (int i = 0; i < 32; ++i) {
+            const bool vis = rw.ok && i < nt[c] && s.pos[c][i] <= rw.qp;
+            const float e = vis ? exp2f(x[i] * b.scale_log2 - rw.m2) : 0.0f;
+            se += e;
+            ne += vis ? 1 : 0;
+            x[i] = e;
           }
+          if (h == 0) {
+            Sc[c] += se;
+            nc[c] += ne;
+          }
+          split_pack32(x, pk);
+          tmem_st32(addr, pk);
         }
         tmem_wait_st();
         tc_fence_before();
@@ -286,16 +282,22 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
         mma_commit(&s.bar);
       }
       const bool last = j == nch - 1;
-      float o[kSub], da[kSub];
-      if (last) load_sub(rw, L.DA, 64 * h, o, da);  // in flight while the MMAs run
+      if (last) stage_half(s, rw, L.DA, h);  // in flight while the MMAs run
       if (!wait_mma(s, phase)) return false;
       if (last) {
+        cp_async_wait_all();  // the thread's own rows of the half buffers
         // ---- epilogue over the 64 channels of half h, kSub at a time
 #pragma unroll 1
         for (int q = 0; q < 64 / kSub; ++q) {
           const int ch0 = 64 * h + kSub * q;
-          float o_n[kSub], da_n[kSub];
-          if (q + 1 < 64 / kSub) load_sub(rw, L.DA, ch0 + kSub, o_n, da_n);
+          float o[kSub], da[kSub];
+#pragma unroll
+          for (int u4 = 0; u4 < kSub / 4; ++u4) {
+            const float4 x = *reinterpret_cast<const float4 *>(&s.oh[threadIdx.x][kSub * q + 4 * u4]);
+            const float4 y = *reinterpret_cast<const float4 *>(&s.dah[threadIdx.x][kSub * q + 4 * u4]);
+            o[4 * u4] = x.x, o[4 * u4 + 1] = x.y, o[4 * u4 + 2] = x.z, o[4 * u4 + 3] = x.w;
+            da[4 * u4] = y.x, da[4 * u4 + 1] = y.y, da[4 * u4 + 2] = y.z, da[4 * u4 + 3] = y.w;
+          }
           uint32_t u[kRound][kSub];
 #pragma unroll
           for (int c = 0; c < kRound; ++c)
@@ -312,6 +314,7 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
               p[0] = da[i];
 #pragma unroll
               for (int T = 1; T < (1 << kRound); ++T) {
+                if (T >= (1 << n)) break;  // subsets of the pass's pages only
                 p[T] = p[T & ~(1 << top_bit(T))] + de[top_bit(T)];
                 ss[T - 1] = fmaf(p[T], p[T], ss[T - 1]);
               }
@@ -331,12 +334,8 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
                 pa[u4] = make_float4(da[4 * u4], da[4 * u4 + 1], da[4 * u4 + 2], da[4 * u4 + 3]);
             }
           }
-#pragma unroll
-          for (int i = 0; i < kSub; ++i) {
-            o[i] = o_n[i];
-            da[i] = da_n[i];
-          }
         }
+        if constexpr (!kScan) __threadfence();  // D_A is read again through L2 by the scan
       }
       // the epilogue's TMEM reads are done before the next MMAs write
       tc_fence_before();
@@ -359,6 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
   for (int i = tid; i < (int)(sizeof(s.q) / 16); i += kThreads) reinterpret_cast<uint4 *>(s.q)[i] = uint4{};
   for (int i = tid; i < (int)(sizeof(s.k) / 16); i += kThreads) reinterpret_cast<uint4 *>(s.k)[i] = uint4{};
   for (int i = tid; i < (int)(sizeof(s.v) / 16); i += kThreads) reinterpret_cast<uint4 *>(&s.v[0][0])[i] = uint4{};
+  for (int i = tid; i < kRows * kHalfPad; i += kThreads) (&s.oh[0][0])[i] = (&s.dah[0][0])[i] = 0.0f;
   if (tid == 0) {
     s.abort_flag = 0;
     mbar_init(&s.bar, 1);
