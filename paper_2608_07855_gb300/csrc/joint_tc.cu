@@ -1,9 +1,11 @@
 // Greedy joint test (Section 3.4, Eq. 11) on the 5th-generation tensor
 // cores: bf16 K/V/Q, head_dim 128, fp32 accumulation in tensor memory.
 //
-// One cooperative persistent kernel, one CTA of 128 threads per SM.  A
-// group is 128 probe rows of one (trajectory, selected layer, KV head):
-// thread i and TMEM lane i hold row i.  In every round (joint_common.cuh) a
+// One cooperative persistent kernel, one CTA of 256 threads per SM.  A
+// group is 128 probe rows of one (trajectory, selected layer, KV head), TMEM
+// lane i holding row i; the CTA's threads form two teams of four warps, and
+// thread i of each team works on row i: the teams split the pages in the
+// softmax and the channels in the epilogue.  In every round (joint_common.cuh) a
 // group makes up to two passes of the same machinery over a list of at
 // most four pages:
 //   fold  the pages of the previous round that were accepted: their D_E are
@@ -44,7 +46,8 @@ using joint::kRound;
 constexpr int D = 128;
 constexpr int kRows = 128;   // probe rows per group (MMA M, TMEM lanes)
 constexpr int kCT = 32;      // page tokens per chunk (the QK N of one page)
-constexpr int kThreads = 128;
+constexpr int kTeam = 128;                 // threads per team (one per row)
+constexpr int kThreads = 2 * kTeam;
 constexpr uint64_t kWait = 1000000000ull;
 constexpr uint32_t kQHalf = kRows * 128;         // one 64-channel half of the Q tile: 16 KB
 constexpr uint32_t kKHalf = kRound * kCT * 128;  // K rows of all pages, one half: 16 KB
@@ -60,6 +63,9 @@ struct SmemJ {
   // row; the padding keeps the rows' 16-byte words in distinct banks)
   alignas(16) float oh[kRows][kHalfPad];
   alignas(16) float dah[kRows][kHalfPad];
+  float Sc[kRound][kRows];     // S_E of every page and row (written by the page's team)
+  int nc[kRound][kRows];       // n_E
+  float part[kCombos + 1][kRows];  // team 1's sums of squares (and ||o||^2) for team 0
   int pos[kRound][kCT];
   unsigned rmax[16];
   uint64_t bar;
@@ -131,15 +137,15 @@ __device__ __forceinline__ bool wait_mma(SmemJ &s, uint32_t &phase) {
 
 constexpr int kSub = 8;  // channels per epilogue step
 
-// Starts the copies of o and D_A of channel half h of the thread's own row
-// into its rows of the half buffers.
+// Starts the copies of o and D_A of the team's 32 channels of half h of the
+// thread's row into that row of the half buffers.
 __device__ __forceinline__ void stage_half(SmemJ &s, const Row &rw, const float *DA, int h) {
   if (!rw.ok) return;
-  const int i = threadIdx.x;
+  const int i = threadIdx.x % kTeam, c0 = 32 * (threadIdx.x / kTeam);
 #pragma unroll
-  for (int u = 0; u < 16; ++u) {
-    cp_async16(&s.oh[i][4 * u], rw.st + 4 + 64 * h + 4 * u);
-    cp_async16(&s.dah[i][4 * u], DA + rw.grow * D + 64 * h + 4 * u);
+  for (int u = 0; u < 8; ++u) {
+    cp_async16(&s.oh[i][c0 + 4 * u], rw.st + 4 + 64 * h + c0 + 4 * u);
+    cp_async16(&s.dah[i][c0 + 4 * u], DA + rw.grow * D + 64 * h + c0 + 4 * u);
   }
 }
 
@@ -154,9 +160,10 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[kSub]) {
 __host__ __device__ constexpr int top_bit(int T) { return T >= 8 ? 3 : T >= 4 ? 2 : T >= 2 ? 1 : 0; }
 
 // One pass over the pages list[0..n) (n <= kRound).  kScan: accumulates the
-// squared norms of the subset sums into ss and o's squared norm into on2;
-// otherwise adds the pages' D_E into D_A in the workspace.  S_E and n_E of
-// each page are left in Sc and nc.  Returns false on a timeout.
+// squared norms of the subset sums over the team's channels into ss, and
+// o's into on2; otherwise adds the pages' D_E into D_A in the workspace.
+// S_E and n_E of every page are left in Sc and nc.  Returns false on a
+// timeout.
 template <bool kScan>
 __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeader *hdr, const Group &G,
                                          const Row &rw, const int *list, int n, bool stage_q, uint32_t tm,
@@ -164,7 +171,7 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
                                          float (&Sc)[kRound], int (&nc)[kRound]) {
   const Batch &b = L.batch;
   const TrajDev &tr = b.t[G.t];
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, team = tid / kTeam, r = tid % kTeam;
   int ps[kRound], pl[kRound];
   int nch = 1;
 #pragma unroll
@@ -236,9 +243,10 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
           mma_commit(&s.bar);
         }
         if (!wait_mma(s, phase)) return false;
-        // ---- e = exp(s - m) on the visible tokens; P over S
+        // ---- e = exp(s - m) on the visible tokens; P over S (team t takes
+        // the pages c = t mod 2)
 #pragma unroll 1
-        for (int c = 0; c < n; ++c) {
+        for (int c = team; c < n; c += 2) {
           float x[32];
           uint32_t pk[32];
           const uint32_t addr = tm + lane_base + kColS + kCT * c;
@@ -257,6 +265,8 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
           if (h == 0) {
             Sc[c] += se;
             nc[c] += ne;
+            s.Sc[c][r] = Sc[c];
+            s.nc[c][r] = nc[c];
           }
           split_pack32(x, pk);
           tmem_st32(addr, pk);
@@ -285,16 +295,24 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
       if (last) stage_half(s, rw, L.DA, h);  // in flight while the MMAs run
       if (!wait_mma(s, phase)) return false;
       if (last) {
-        cp_async_wait_all();  // the thread's own rows of the half buffers
-        // ---- epilogue over the 64 channels of half h, kSub at a time
+        cp_async_wait_all();  // the thread's own parts of the half buffers
+        if (h == 0) {
+#pragma unroll
+          for (int c = 0; c < kRound; ++c)
+            if (c < n) {
+              Sc[c] = s.Sc[c][r];
+              nc[c] = s.nc[c][r];
+            }
+        }
+        // ---- epilogue over the team's 32 channels of half h, kSub at a time
 #pragma unroll 1
-        for (int q = 0; q < 64 / kSub; ++q) {
+        for (int q = 4 * team; q < 4 * team + 4; ++q) {
           const int ch0 = 64 * h + kSub * q;
           float o[kSub], da[kSub];
 #pragma unroll
           for (int u4 = 0; u4 < kSub / 4; ++u4) {
-            const float4 x = *reinterpret_cast<const float4 *>(&s.oh[threadIdx.x][kSub * q + 4 * u4]);
-            const float4 y = *reinterpret_cast<const float4 *>(&s.dah[threadIdx.x][kSub * q + 4 * u4]);
+            const float4 x = *reinterpret_cast<const float4 *>(&s.oh[r][kSub * q + 4 * u4]);
+            const float4 y = *reinterpret_cast<const float4 *>(&s.dah[r][kSub * q + 4 * u4]);
             o[4 * u4] = x.x, o[4 * u4 + 1] = x.y, o[4 * u4 + 2] = x.z, o[4 * u4 + 3] = x.w;
             da[4 * u4] = y.x, da[4 * u4 + 1] = y.y, da[4 * u4 + 2] = y.z, da[4 * u4 + 3] = y.w;
           }
@@ -372,7 +390,8 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tm = s.tmem;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  // warps w and w + 4 (the two teams) reach TMEM lanes 32 (w mod 4) ..
+  const uint32_t lane_base = (uint32_t)((warp % 4) * 32) << 16;
   uint32_t phase = 0;
   bool ok = true;
 
@@ -398,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
       for (int c = 0; c < kc; ++c) cand[c] = L.cand[G.t][r * kRound + c];
 
       Row rw;
-      const int row = G.row0 + tid;
+      const int row = G.row0 + tid % kTeam;
       rw.ok = row < G.rows;
       const int hq = G.kvh * b.g + (rw.ok ? row / tr.W : 0), w = rw.ok ? row % tr.W : 0;
       rw.grow = L.row_off[G.t] + (int64_t)(G.li * b.H + G.kvh) * G.rows + (rw.ok ? row : 0);
@@ -427,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
             rw.SA += Sc[c];
             rw.nA += nc[c];
           }
-        if (rw.ok) {
+        if (rw.ok && tid < kTeam) {
           L.SA[rw.grow * 2] = rw.SA;
           L.SA[rw.grow * 2 + 1] = (float)rw.nA;
         }
@@ -436,23 +455,35 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
         ok = false;
         break;
       }
-      // Eq. 6 on A u T for every non-empty subset T of the round's pages;
-      // S and n added in candidate order
-      const float onorm = sqrtf(on2);
+      // team 1's channel sums to team 0
+      if (tid >= kTeam) {
 #pragma unroll
-      for (int T = 1; T < (1 << kRound); ++T) {
-        if (T >= (1 << kc)) break;
-        float S_tot = rw.SA;
-        int n_tot = rw.nA;
+        for (int i = 0; i < kCombos; ++i) s.part[i][tid - kTeam] = ss[i];
+        s.part[kCombos][tid - kTeam] = on2;
+      }
+      __syncthreads();
+      if (tid < kTeam) {
 #pragma unroll
-        for (int c = 0; c < kRound; ++c)
-          if ((T >> c) & 1) {
-            S_tot += Sc[c];
-            n_tot += nc[c];
-          }
-        const float rv = rw.ok ? effect_value(n_tot, rw.nvis, S_tot, rw.l, ss[T - 1], onorm) : 0.0f;
-        const unsigned mx = __reduce_max_sync(0xffffffffu, __float_as_uint(rv));
-        if (lane == 0) atomicMax(&s.rmax[T - 1], mx);
+        for (int i = 0; i < kCombos; ++i) ss[i] += s.part[i][tid];
+        on2 += s.part[kCombos][tid];
+        // Eq. 6 on A u T for every non-empty subset T of the round's pages;
+        // S and n added in candidate order
+        const float onorm = sqrtf(on2);
+#pragma unroll
+        for (int T = 1; T < (1 << kRound); ++T) {
+          if (T >= (1 << kc)) break;
+          float S_tot = rw.SA;
+          int n_tot = rw.nA;
+#pragma unroll
+          for (int c = 0; c < kRound; ++c)
+            if ((T >> c) & 1) {
+              S_tot += Sc[c];
+              n_tot += nc[c];
+            }
+          const float rv = rw.ok ? effect_value(n_tot, rw.nvis, S_tot, rw.l, ss[T - 1], onorm) : 0.0f;
+          const unsigned mx = __reduce_max_sync(0xffffffffu, __float_as_uint(rv));
+          if (lane == 0) atomicMax(&s.rmax[T - 1], mx);
+        }
       }
       __syncthreads();
       if (tid < (1 << kc) - 1) atomic_max_nonneg(tab_r + G.t * kCombos + tid, __uint_as_float(s.rmax[tid]));
