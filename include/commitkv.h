@@ -330,6 +330,33 @@ commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
                                  void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Compression checkpoint in place, Section 3.4, Eq. 12-13 and Eq. 4.
+ *
+ * The selection of commitkv_compact (same arguments and rules, same idx_out
+ * and n_idx_out), with the gather done inside the cache: K and V row I_j of
+ * every (layer, KV head) slice moves to row j of the same slice, in the
+ * cache's own layout and strides, and pos[j] = pos[I_j], for j < |I_j|.  The
+ * cache's k, v and pos buffers are overwritten (their const in
+ * commitkv_traj notwithstanding); rows and positions at and after |I_j| keep
+ * stale values, and the caller's cache length becomes |I_j|.  No second
+ * cache-sized buffer is needed.  Because I_j is strictly increasing with
+ * I_j >= j, the rows are moved in ascending chunks, each read whole before
+ * any of its rows is written.
+ *
+ *   cache        the caches to compact: k, v and pos must be non-NULL when
+ *                S_t > 0 (else COMMITKV_ERR_INVALID_ARG).
+ *   other arguments as for commitkv_compact.
+ * -------------------------------------------------------------------- */
+commitkv_status commitkv_compact_in_place(const commitkv_shape *shape, int32_t n_traj,
+                                          const commitkv_traj *cache, const uint8_t *const *retired,
+                                          const int32_t *const *pending, const int32_t *n_pending,
+                                          const float *const *pending_priority,
+                                          const float *const *fill_score, int32_t budget_B,
+                                          int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                          int32_t *const *idx_out, int32_t *n_idx_out, void *workspace,
+                                          size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * commitkv_compact without a workspace.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory where
  * they compact.  A serving engine usually reserves nearly all device memory

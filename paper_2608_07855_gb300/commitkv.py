@@ -93,12 +93,14 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
                                         vp, vp, vp, sz, vp]
     lib.commitkv_compact.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, i32, i32, i32,
                                      vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.commitkv_compact_in_place.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, i32, i32, i32,
+                                              vp, vp, vp, sz, vp]
     lib.commitkv_compact_noalloc.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, i32, i32,
                                              i32, vp, vp, vp, vp, vp, vp, vp]
     lib.commitkv_test_barrier_timeout.argtypes = [vp, sz, i32, vp]
     for f in ("commitkv_workspace_init", "commitkv_workspace_status", "commitkv_page_effects",
               "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_classify_variant", "commitkv_joint_test", "commitkv_compact",
-              "commitkv_compact_noalloc", "commitkv_test_barrier_timeout"):
+              "commitkv_compact_in_place", "commitkv_compact_noalloc", "commitkv_test_barrier_timeout"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -334,6 +336,24 @@ def commitkv_compact(shape: Shape, cache, retired, pending, pending_priority, fi
         _ptr_array(idx_out, n), _ptr(n_idx_out), _ptr_array(k_out, n), _ptr_array(v_out, n),
         _ptr_array(pos_out, n), _ptr(workspace), workspace.numel(), _stream(stream))
     _check(rc, "commitkv_compact")
+
+
+def commitkv_compact_in_place(shape: Shape, cache, retired, pending, pending_priority, fill_score, budget_B,
+                              pending_tokens_BN, pending_cap_pages, idx_out, n_idx_out, workspace=None,
+                              stream=None):
+    """commitkv_compact with the gather inside the caches: K and V row I_j
+    of every (layer, KV head) slice moves to row j of the same slice, and
+    pos[j] = pos[I_j], for j < n_idx_out[t]; the caches' k, v and pos
+    tensors are overwritten."""
+    n = len(cache)
+    d = _descs(cache)
+    npend = (ctypes.c_int32 * n)(*[0 if p is None else int(p.numel()) for p in pending])
+    rc = load_library().commitkv_compact_in_place(
+        ctypes.byref(shape), n, d, _ptr_array(retired, n), _ptr_array(pending, n),
+        ctypes.cast(npend, ctypes.c_void_p), _ptr_array(pending_priority, n),
+        _ptr_array(fill_score, n), int(budget_B), int(pending_tokens_BN), int(pending_cap_pages),
+        _ptr_array(idx_out, n), _ptr(n_idx_out), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(rc, "commitkv_compact_in_place")
 
 
 def commitkv_compact_noalloc(shape: Shape, cache, retired, pending, pending_priority, fill_score,

@@ -556,7 +556,7 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
   return cuda_status(launch_joint(L, hdr, stream, sms));
 }
 
-commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
+static commitkv_status compact_impl(const commitkv_shape *shape, int32_t n_traj,
                                  const commitkv_traj *cache, const uint8_t *const *retired,
                                  const int32_t *const *pending, const int32_t *n_pending,
                                  const float *const *pending_priority,
@@ -564,7 +564,8 @@ commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
                                  int32_t pending_tokens_BN, int32_t pending_cap_pages,
                                  int32_t *const *idx_out, int32_t *n_idx_out,
                                  void *const *k_out, void *const *v_out, int32_t *const *pos_out,
-                                 void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+                                 void *workspace, size_t workspace_bytes, cudaStream_t stream,
+                                   bool in_place) {
   commitkv_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_trajs(shape, n_traj, cache, false))) return st;
@@ -606,7 +607,38 @@ commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
   L.B = budget_B;
   L.B_N = pending_tokens_BN;
   L.cap = pending_cap_pages;
+  L.in_place = in_place ? 1 : 0;
   return cuda_status(launch_compact(L, static_cast<WsHeader *>(workspace), stream));
+}
+
+commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
+                                 const commitkv_traj *cache, const uint8_t *const *retired,
+                                 const int32_t *const *pending, const int32_t *n_pending,
+                                 const float *const *pending_priority,
+                                 const float *const *fill_score, int32_t budget_B,
+                                 int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                 int32_t *const *idx_out, int32_t *n_idx_out,
+                                 void *const *k_out, void *const *v_out, int32_t *const *pos_out,
+                                 void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+  return compact_impl(shape, n_traj, cache, retired, pending, n_pending, pending_priority, fill_score, budget_B,
+                      pending_tokens_BN, pending_cap_pages, idx_out, n_idx_out, k_out, v_out, pos_out, workspace,
+                      workspace_bytes, stream, false);
+}
+
+commitkv_status commitkv_compact_in_place(const commitkv_shape *shape, int32_t n_traj,
+                                          const commitkv_traj *cache, const uint8_t *const *retired,
+                                          const int32_t *const *pending, const int32_t *n_pending,
+                                          const float *const *pending_priority,
+                                          const float *const *fill_score, int32_t budget_B,
+                                          int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                          int32_t *const *idx_out, int32_t *n_idx_out, void *workspace,
+                                          size_t workspace_bytes, cudaStream_t stream) {
+  if (!cache) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj && t < COMMITKV_MAX_TRAJ; ++t)
+    if (cache[t].S > 0 && (!cache[t].k || !cache[t].v || !cache[t].pos)) return COMMITKV_ERR_INVALID_ARG;
+  return compact_impl(shape, n_traj, cache, retired, pending, n_pending, pending_priority, fill_score, budget_B,
+                      pending_tokens_BN, pending_cap_pages, idx_out, n_idx_out, nullptr, nullptr, nullptr,
+                      workspace, workspace_bytes, stream, true);
 }
 
 }  // extern "C"

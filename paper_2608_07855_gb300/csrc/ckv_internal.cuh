@@ -176,6 +176,7 @@ struct CompactLaunch {
   void *v_out[kMaxTraj];
   int32_t *pos_out[kMaxTraj];
   int32_t B, B_N, cap;
+  int32_t in_place;  // gather into the cache itself (rows 0..|I|-1 of every slice)
 };
 cudaError_t launch_compact(const CompactLaunch &L, WsHeader *hdr, cudaStream_t stream);
 

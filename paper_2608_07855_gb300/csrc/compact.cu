@@ -5,7 +5,10 @@
 //         pending prefix, pick the fill tokens by an exact radix select on
 //         64-bit keys (fill score, token index), and write I_j ascending;
 // gather  16-byte vector copies of the retained K and V rows of every
-//         (layer, KV head), plus positions.
+//         (layer, KV head), plus positions; into caller buffers, or in place
+//         (the retained rows move to rows 0..|I|-1 of the cache itself).
+#include <type_traits>
+
 #include "ckv_internal.cuh"
 
 namespace ckv {
@@ -248,6 +251,65 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Com
   if (slice == 0 && vv == 0 && L.pos_out[t]) L.pos_out[t][j] = tr.pos[i];
 }
 
+// In-place gather: one block per (K or V, layer, KV head, trajectory)
+// slice.  I is strictly increasing with I_j >= j, so row j's destination is
+// a source only for rows k <= j.  The block walks the slice in chunks of
+// ROWS rows: it reads every source row of the chunk, waits at the barrier,
+// then writes the chunk's destinations.  A destination in chunk c is read,
+// if at all, by a row of chunk c or earlier, before that chunk's barrier;
+// sources of later chunks lie at or after their own rows, past every row
+// written so far.  Rows with I_j = j are left alone.
+template <int VEC_BYTES, int ROWS>
+__global__ void __launch_bounds__(256) gather_in_place_kernel(const __grid_constant__ CompactLaunch L) {
+  using Vec = typename std::conditional<VEC_BYTES == 16, uint4, uint16_t>::type;
+  constexpr int kMaxVec = 512 / VEC_BYTES;  // vectors per row at most (fp32, d = 128)
+  constexpr int kPer = ROWS * kMaxVec / 256;
+  const int t = blockIdx.z, slice = blockIdx.y;
+  const TrajDev &tr = L.t[t];
+  const int l = slice / L.H, h = slice % L.H;
+  const int vpr = L.d * L.elem_bytes / VEC_BYTES;
+  char *base = static_cast<char *>(const_cast<void *>(blockIdx.x ? tr.v : tr.k)) +
+               ((int64_t)l * tr.sl + (int64_t)h * tr.sh) * L.elem_bytes;
+  const int64_t rs = tr.st * L.elem_bytes;
+  const int n = L.n_idx[t];
+  const int32_t *idx = L.idx[t];
+  for (int j0 = 0; j0 < n; j0 += ROWS) {
+    Vec buf[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int e = threadIdx.x + 256 * u, r = e / vpr, w = e % vpr;
+      if (r < ROWS && j0 + r < n) {
+        const int i = idx[j0 + r];
+        if (i != j0 + r) buf[u] = *reinterpret_cast<const Vec *>(base + i * rs + w * VEC_BYTES);
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int e = threadIdx.x + 256 * u, r = e / vpr, w = e % vpr;
+      if (r < ROWS && j0 + r < n) {
+        const int i = idx[j0 + r];
+        if (i != j0 + r) *reinterpret_cast<Vec *>(base + (int64_t)(j0 + r) * rs + w * VEC_BYTES) = buf[u];
+      }
+    }
+  }
+}
+
+// Positions in place, one block per trajectory, by the same chunk rule.
+__global__ void __launch_bounds__(256) positions_in_place_kernel(const __grid_constant__ CompactLaunch L) {
+  const int t = blockIdx.x;
+  int32_t *pos = const_cast<int32_t *>(L.t[t].pos);
+  const int n = L.n_idx[t];
+  const int32_t *idx = L.idx[t];
+  for (int j0 = 0; j0 < n; j0 += 256) {
+    const int j = j0 + threadIdx.x;
+    int v = 0;
+    if (j < n) v = pos[idx[j]];
+    __syncthreads();
+    if (j < n) pos[j] = v;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_compact(const CompactLaunch &L, WsHeader *hdr, cudaStream_t stream) {
@@ -255,6 +317,23 @@ cudaError_t launch_compact(const CompactLaunch &L, WsHeader *hdr, cudaStream_t s
   select_kernel<<<L.n_traj, kThreads, 0, stream>>>(L, hdr);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (L.in_place) {
+    bool aligned = (L.d * L.elem_bytes) % 16 == 0;
+    for (int t = 0; t < L.n_traj; ++t) {
+      const TrajDev &tr = L.t[t];
+      aligned &= ((uintptr_t)tr.k % 16 == 0) && ((uintptr_t)tr.v % 16 == 0) &&
+                 ((tr.sl * L.elem_bytes) % 16 == 0) && ((tr.sh * L.elem_bytes) % 16 == 0) &&
+                 ((tr.st * L.elem_bytes) % 16 == 0);
+    }
+    if (L.B == 0) return cudaSuccess;
+    dim3 grid(2, L.M * L.H, L.n_traj);
+    if (aligned) gather_in_place_kernel<16, 64><<<grid, 256, 0, stream>>>(L);
+    else gather_in_place_kernel<2, 8><<<grid, 256, 0, stream>>>(L);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    positions_in_place_kernel<<<L.n_traj, 256, 0, stream>>>(L);
+    return cudaGetLastError();
+  }
   bool any_out = false;
   bool aligned = (L.d * L.elem_bytes) % 16 == 0;
   for (int t = 0; t < L.n_traj; ++t) {

@@ -11,12 +11,13 @@ library's entry points in the order of Algorithm 1:
   pre_commit   commit c_t: R- of every resident page over the pre-commit
                window (commitkv_page_effects); the non-retired pages form
                E_{c_t} and wait for their post-commit measurement.
-  checkpoint   commitkv_compact: the retired pages D_c are dropped, at most
-               B_N = floor(eta B) tokens / protect_cap pages of the waiting
-               pages are kept by decreasing R- (Eq. 12), the budget B is
-               filled by the caller's per-token score (Eq. 13), and K, V and
-               positions are gathered (Eq. 4); page spans are found again from
-               the retained indices (a page keeps whichever of its tokens are
+  checkpoint   commitkv_compact_in_place: the retired pages D_c are
+               dropped, at most B_N = floor(eta B) tokens / protect_cap pages
+               of the waiting pages are kept by decreasing R- (Eq. 12), the
+               budget B is filled by the caller's per-token score (Eq. 13),
+               and K, V and positions are gathered (Eq. 4) inside the
+               session's own buffers; page spans are found again from the
+               retained indices (a page keeps whichever of its tokens are
                retained, which stay contiguous).
   post_commit  R+ over the post-commit window with the row stats;
                classification (Eq. 9-10, or an ablation variant of Section
@@ -140,19 +141,12 @@ class Session:
         prio_p = torch.zeros(max(P, 1), dtype=torch.float32, device=self.dev)
         if P:
             prio_p[:P] = torch.tensor([self.R_pre.get(pid, 0.0) for pid in ids], dtype=torch.float32)
-        M, H, d = self.shape.layers, self.shape.kv_heads, self.shape.head_dim
         idx = torch.full((max(B, 1),), -1, dtype=torch.int32, device=self.dev)
         n_idx = torch.zeros(1, dtype=torch.int32, device=self.dev)
-        k_out = torch.empty(M, H, B, d, dtype=self.K.dtype, device=self.dev)
-        v_out = torch.empty(M, H, B, d, dtype=self.V.dtype, device=self.dev)
-        pos_out = torch.empty(max(B, 1), dtype=torch.int32, device=self.dev)
-        ck.commitkv_compact(self.shape, [tr], [retired], [pending], [prio_p], [fill[:self.S]], B, self.B_N,
-                            self.protect_cap, [idx], n_idx, [k_out], [v_out], [pos_out], workspace=ws)
+        ck.commitkv_compact_in_place(self.shape, [tr], [retired], [pending], [prio_p], [fill[:self.S]], B,
+                                     self.B_N, self.protect_cap, [idx], n_idx, workspace=ws)
         self._check()
         n = int(n_idx[0])
-        self.K[:, :, :n].copy_(k_out[:, :, :n])
-        self.V[:, :, :n].copy_(v_out[:, :, :n])
-        self.pos[:n].copy_(pos_out[:n])
         I = idx[:n].cpu().tolist()
         # page spans from the retained indices
         new_index = {old: new for new, old in enumerate(I)}

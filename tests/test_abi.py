@@ -17,7 +17,7 @@ def lib():
 def test_header_declares_the_entry_points():
     names = ck.declared_functions()
     for n in ("commitkv_page_effects", "commitkv_classify", "commitkv_joint_test", "commitkv_compact",
-              "commitkv_workspace_size", "commitkv_workspace_init", "commitkv_workspace_status",
+              "commitkv_compact_in_place", "commitkv_workspace_size", "commitkv_workspace_init", "commitkv_workspace_status",
               "commitkv_status_string"):
         assert n in names
 
@@ -94,6 +94,23 @@ def test_classify_and_compact_validation(lib):
     npend = (ctypes.c_int32 * 1)(100000)
     assert lib.commitkv_compact(ctypes.byref(shape), 1, trajs, ptrs, ptrs, npend, ptrs, ptrs, 10, 5, 4,
                                 ptrs, 0x3000, None, None, None, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
+
+
+def test_compact_in_place_validation(lib):
+    """The in-place checkpoint checks its arguments like commitkv_compact and
+    needs the cache's K, V and positions (it writes them)."""
+    ptrs = (ctypes.c_void_p * 1)(0x1000)
+    shape = ck.Shape(2, 2, 8, 128, ck.COMMITKV_BF16, 0.0)
+    npend = (ctypes.c_int32 * 1)(0)
+    trajs = (ck.Traj * 1)(_good_traj())
+    # B_N > B
+    assert lib.commitkv_compact_in_place(ctypes.byref(shape), 1, trajs, ptrs, None, npend, None, ptrs, 10, 11, 4,
+                                         ptrs, 0x3000, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
+    # no K to compact
+    bad = _good_traj()
+    bad.k = None
+    assert lib.commitkv_compact_in_place(ctypes.byref(shape), 1, (ck.Traj * 1)(bad), ptrs, None, npend, None, ptrs,
+                                         10, 5, 4, ptrs, 0x3000, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
 
 
 def test_workspace_covers_smaller_caches(lib):

@@ -298,6 +298,54 @@ def test_compact_isolated(name, seed):
     assert np.array_equal(_np(b.pos_out[0])[:n], pw)
 
 
+@pytest.mark.parametrize("layout", ["capacity", "odd_offset"])
+@pytest.mark.parametrize("name,seed", CASES)
+def test_compact_in_place(name, seed, layout):
+    """commitkv_compact_in_place on a copy of the cache kept inside a larger
+    buffer: I_j as the oracle's, and rows / positions [0, |I_j|) of the cache
+    itself bit-exact against the oracle's gathered K~, V~, p~; memory
+    outside the cache's view untouched.  'capacity': the cache is the first
+    S tokens of a buffer with room for more (16-byte vector path);
+    'odd_offset': every row starts one element into a row of d + 1 (the
+    unaligned path)."""
+    r = get_run(name, seed)
+    cfg, b, dev, o, tr = r.cfg, r.buf, r.dev, r.orc, r.tr
+    retired = torch.from_numpy(o.accepted.astype(np.uint8)).cuda()
+    prio = torch.from_numpy(o.R_post32).cuda()
+    M, H, S, d = dev.K.shape
+    if layout == "capacity":
+        Kb = torch.zeros(M, H, S + 37, d, dtype=dev.K.dtype, device="cuda")
+        Vb = torch.zeros_like(Kb)
+        K, V = Kb[:, :, :S], Vb[:, :, :S]
+    else:
+        Kb = torch.zeros(M, H, S, d + 1, dtype=dev.K.dtype, device="cuda")
+        Vb = torch.zeros_like(Kb)
+        K, V = Kb[..., 1:], Vb[..., 1:]
+    K.copy_(dev.K)
+    V.copy_(dev.V)
+    pos = dev.pos.clone()
+    cache = ck.TrajTensors(K, V, pos, dev.Q_post, dev.qpos_post, dev.page_start, dev.page_len)
+    idx = torch.full_like(b.idx[0], -1)
+    n_idx = torch.zeros_like(b.n_idx)
+    ck.commitkv_compact_in_place(b.shape, [cache], [retired], [dev.pending], [prio], [dev.fill], cfg.B, cfg.B_N,
+                                 cfg.pending_cap, [idx], n_idx, workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    n = int(n_idx[0])
+    assert n == len(o.I)
+    assert np.array_equal(_np(idx)[:n], o.I)
+    Kw, Vw, pw = core.gather(tr.K, tr.V, tr.pos, o.I)
+    kg, vg = K[:, :, :n], V[:, :, :n]
+    if cfg.dtype == "bf16":
+        kg, vg = kg.view(torch.uint16), vg.view(torch.uint16)
+    assert np.array_equal(_np(kg), Kw) and np.array_equal(_np(vg), Vw)
+    assert np.array_equal(_np(pos)[:n], pw)
+    if layout == "capacity":
+        assert not Kb[:, :, S:].any() and not Vb[:, :, S:].any()
+    else:
+        assert not Kb[..., 0].any() and not Vb[..., 0].any()
+
+
 @pytest.mark.parametrize("name,seed", [("tiny", 0), ("small", 1), ("small_f32", 3)])
 def test_full_step(name, seed):
     """The whole launch sequence of one step: every decision of the GPU
