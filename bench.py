@@ -35,13 +35,9 @@ PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum, one ncu pass) of
 # one scoring call of a step (prep + pass A + combine + pass B over the pre-
-# and post-commit caches), full-size workload, with the sha256 prefix of the
-# scoring sources they were taken with: reported only while those sources are
-# unchanged.
-# DRAM bytes of the scoring call per step (ncu dram__bytes_read.sum +
-# dram__bytes_write.sum of prep, pass A, combine and pass B): the 4-layer
-# slice of the workload captured, times 9 (36 layers); keyed by the
-# scoring sources it was measured on.
+# and post-commit caches): the 4-layer slice of the workload captured, times 9
+# (36 layers), with the sha256 prefix of the scoring sources it was taken
+# with; reported only while those sources are unchanged.
 MEASURED_TRAFFIC = {"qwen3_8b_32k": (18748523520, "dbb1f9af1c7b3530")}
 TRAFFIC_SOURCES = ("score_tc.cu", "score_tc.cuh", "sm103.cuh")
 
