@@ -16,18 +16,19 @@
 //         T of them, max over the rows (Eq. 7) into the round's table.
 // A pass stages Q (once per group and round) and the pages' K and V rows in
 // shared memory (cp.async into the 128-byte-swizzled layout) and issues
-//   S = Q K^T       one MMA chain with N = 64 x pages, TMEM columns 256..511
+//   S = Q K^T       one MMA chain with N = 32 x pages, TMEM columns 256..383
 //   e = exp(s - m)  per row on the page's visible tokens (m = the row's
 //                   final max); S_E = sum e, n_E = count; P = e written
 //                   over S as a bf16 (hi, lo) pair
 //   U_E = P V_E     per page and 64-channel half, TMEM columns 64 c, TS form
 //                   (P from tensor memory, V from shared memory)
-// and the epilogue reads U_E 16 columns at a time: D_E = U_E - S_E o.  In
+// and the epilogue reads U_E 8 columns at a time (o and D_A of the channel
+// half staged in shared memory while the MMAs run): D_E = U_E - S_E o.  In
 // the scan the sums of the subsets are built as a tree in which every
 // subset adds its largest page last, so each is the sum that the
 // one-page-at-a-time scan forms, ((D_A + D_b1) + D_b2) + ... + D_c, and its
 // squared norm accumulates over the channels in order.
-// Pages longer than 64 tokens are taken in 64-token chunks: U accumulates
+// Pages longer than 32 tokens are taken in 32-token chunks: U accumulates
 // over the chunks, and the chunks' QK and softmax are redone for the second
 // channel half.  Every mbarrier wait is bounded (1 s); on expiry the kernel
 // records COMMITKV_ERR_TIMEOUT, raises the abort flag that the grid barrier
