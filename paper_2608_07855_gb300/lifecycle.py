@@ -25,6 +25,10 @@ library's entry points in the order of Algorithm 1:
                most 64 pages per commit); the greedy joint test (Eq. 11);
                D_c gains the accepted pages.
 
+state_dict / load_state_dict carry the state between commits (the resident
+cache, the page table, R- of the latest pre-commit, the pages waiting for
+their post-commit measurement, D_c) for checkpoint and resume.
+
 Every computation runs in the library's kernels; this module keeps the page
 table and the buffers.  The host reads back small per-commit results (page
 effects, candidate counts, accepted masks, retained indices) to keep the page
@@ -86,6 +90,47 @@ class Session:
 
     def page_ids(self):
         return [p[0] for p in self.pages]
+
+    # ---------------------------------------------------------------- resume
+    def state_dict(self):
+        """Everything the session carries from one commit to the next: the
+        resident cache (K, V, positions of its S tokens), the page table, R-
+        of the latest pre-commit, the pages waiting for their post-commit
+        measurement and D_c.  Tensors are copies on the session's device;
+        torch.save writes the dict."""
+        S = self.S
+        return {
+            "config": self._config(),
+            "K": self.K[:, :, :S].clone(), "V": self.V[:, :, :S].clone(), "pos": self.pos[:S].clone(),
+            "pages": [list(p) for p in self.pages], "next_id": self.next_id,
+            "R_pre": dict(self.R_pre), "measured": list(self.measured), "retired": sorted(self.retired),
+        }
+
+    def load_state_dict(self, st):
+        """Resumes from state_dict() of a session with the same model shape,
+        page size, budget and decision settings; the resident cache must fit
+        this session's capacity."""
+        if st["config"] != self._config():
+            raise ValueError("state of a session with other settings")
+        S = int(st["pos"].shape[0])
+        if S > self.cap:
+            raise ValueError("session capacity exceeded")
+        self.K[:, :, :S].copy_(st["K"])
+        self.V[:, :, :S].copy_(st["V"])
+        self.pos[:S].copy_(st["pos"])
+        self.S = S
+        self.pages = [list(p) for p in st["pages"]]
+        self.next_id = int(st["next_id"])
+        self.R_pre = dict(st["R_pre"])
+        self.measured = list(st["measured"])
+        self.retired = set(st["retired"])
+
+    def _config(self):
+        s, th = self.shape, self.thresholds
+        return {"shape": (s.layers, s.kv_heads, s.q_heads, s.head_dim, s.dtype, float(s.softmax_scale)),
+                "G": self.G, "B": self.B, "B_N": self.B_N, "scan_cap": self.scan_cap,
+                "protect_cap": self.protect_cap, "variant": int(self.variant), "tau_joint": float(self.tau_joint),
+                "thresholds": None if th is None else (th.tau_use, th.tau_dead, th.rho_use, th.rho_dead)}
 
     # ---------------------------------------------------------------- cache
     def append(self, K, V, pos, events):
