@@ -557,15 +557,15 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
 }
 
 static commitkv_status compact_impl(const commitkv_shape *shape, int32_t n_traj,
-                                 const commitkv_traj *cache, const uint8_t *const *retired,
-                                 const int32_t *const *pending, const int32_t *n_pending,
-                                 const float *const *pending_priority,
-                                 const float *const *fill_score, int32_t budget_B,
-                                 int32_t pending_tokens_BN, int32_t pending_cap_pages,
-                                 int32_t *const *idx_out, int32_t *n_idx_out,
-                                 void *const *k_out, void *const *v_out, int32_t *const *pos_out,
-                                 void *workspace, size_t workspace_bytes, cudaStream_t stream,
-                                   bool in_place) {
+                                    const commitkv_traj *cache, const uint8_t *const *retired,
+                                    const int32_t *const *pending, const int32_t *n_pending,
+                                    const float *const *pending_priority,
+                                    const float *const *fill_score, int32_t budget_B,
+                                    int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                    int32_t *const *idx_out, int32_t *n_idx_out,
+                                    void *const *k_out, void *const *v_out, int32_t *const *pos_out,
+                                    void *workspace, size_t workspace_bytes, cudaStream_t stream,
+                                    bool in_place) {
   commitkv_status st = check_shape(shape);
   if (st) return st;
   if ((st = check_trajs(shape, n_traj, cache, false))) return st;
