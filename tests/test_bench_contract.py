@@ -35,8 +35,14 @@ def test_launches_per_step():
 
 
 def test_peaks_are_the_measured_ones():
+    """The denominators are the measured peaks when the measurement file is
+    there, else the documented fallback."""
     peaks, kind = bench.load_peaks()
-    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if not os.path.exists(path):
+        assert kind == "fallback" and peaks == bench.PEAKS_FALLBACK
+        return
+    with open(path) as f:
         m = json.load(f)
     assert kind == "measured"
     assert peaks["hbm_gbs"] == m["hbm_gbs"] and peaks["bf16_tflops_sustained"] == m["bf16_tflops_sustained"]
