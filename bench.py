@@ -82,6 +82,18 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(value: float, world: int, device) -> float:
+    """The largest of the ranks' values: the job's timed region ends with its
+    slowest rank.  The value itself at world size 1."""
+    if world <= 1:
+        return value
+    import torch
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 class Clocks:
     """nvidia-smi sampling during the timed region."""
 
@@ -254,10 +266,7 @@ def run_ours(args, rank, world, local):
     st = buf.status()
     if st != ck.COMMITKV_OK:
         raise RuntimeError(f"device status after timing: {ck.status_string(st)}")
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, "cuda")
     ms_per_step = total_ms / args.steps
     value = tokens_per_step * world / (ms_per_step / 1e3)
 
@@ -412,11 +421,7 @@ def run_e2e(args, cfg, trs, devs, buf, tokens_per_step, world):
     compute.wait_stream(copy)
     t1.record(compute)
     torch.cuda.synchronize()
-    ms = t0.elapsed_time(t1) / steps
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t0.elapsed_time(t1) / steps, world, "cuda")
     return {"value": tokens_per_step * world / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
             "steps": steps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "upload_overlapped": ns > 1}
