@@ -113,6 +113,40 @@ def test_compact_in_place_validation(lib):
                                          10, 5, 4, ptrs, 0x3000, 0x90000, 1 << 20, None) == ck.COMMITKV_ERR_INVALID_ARG
 
 
+def test_joint_and_variant_validation(lib):
+    """Host checks of the joint test, the from-stats scoring and the
+    classify variants: nothing is launched on a bad argument."""
+    shape = ck.Shape(2, 2, 8, 128, ck.COMMITKV_BF16, 0.0)
+    trajs = (ck.Traj * 1)(_good_traj())
+    ptrs = (ctypes.c_void_p * 1)(0x1000)
+    n_cand = 0x2000
+    jt = lib.commitkv_joint_test
+    # tau_joint NaN
+    assert jt(ctypes.byref(shape), 1, trajs, None, ptrs, ptrs, n_cand, float("nan"), ptrs, None, 0x90000, 1 << 30,
+              None) == ck.COMMITKV_ERR_INVALID_ARG
+    # no stats / no candidates / no accepted output
+    for st, cd, acc in ((None, ptrs, ptrs), (ptrs, None, ptrs), (ptrs, ptrs, None)):
+        assert jt(ctypes.byref(shape), 1, trajs, None, st, cd, n_cand, 0.05, acc, None, 0x90000, 1 << 30,
+                  None) == ck.COMMITKV_ERR_INVALID_ARG
+    # workspace too small
+    assert jt(ctypes.byref(shape), 1, trajs, None, ptrs, ptrs, n_cand, 0.05, ptrs, None, 0x90000, 4096,
+              None) == ck.COMMITKV_ERR_WORKSPACE
+    # the from-stats scoring needs its stats
+    R = (ctypes.c_void_p * 1)(0x80000)
+    assert lib.commitkv_page_effects_from_stats(ctypes.byref(shape), 1, trajs, None, None, R, None, 0x90000, 1 << 30,
+                                                None) == ck.COMMITKV_ERR_INVALID_ARG
+    # classify variants: unknown bits
+    P = (ctypes.c_int32 * 1)(10)
+    th = ck.Thresholds(0.05, 0.01, 0.75, 0.25)
+    cv = lib.commitkv_classify_variant
+    assert cv(1, P, ptrs, ptrs, ptrs, ctypes.byref(th), 4, ptrs, ptrs, 0x2000, 0x90000, 1 << 20,
+              None) == ck.COMMITKV_ERR_INVALID_ARG
+    # a negative page count
+    Pn = (ctypes.c_int32 * 1)(-1)
+    assert cv(1, Pn, ptrs, ptrs, ptrs, ctypes.byref(th), 0, ptrs, ptrs, 0x2000, 0x90000, 1 << 20,
+              None) == ck.COMMITKV_ERR_INVALID_ARG
+
+
 def test_workspace_covers_smaller_caches(lib):
     """A workspace sized for the post-commit caches serves the pre-commit
     call too (its S and P are smaller), for every chunking regime."""
