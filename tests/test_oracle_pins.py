@@ -173,6 +173,31 @@ def test_uniform_attention_textbook():
             assert _close(R_head[0, h, E], want, 1e-12), (h, E)
 
 
+def test_row_stats_textbook():
+    """The row statistics every closed form and the GPU's stats outputs rest
+    on, against a softmax written out row by row: m = max of the scaled
+    scores of the visible tokens, l = sum exp(s - m), o = the attention
+    output, n = the visible count (query head h reads KV head h // g)."""
+    rng = np.random.default_rng(21)
+    pb = _random_problem(rng, M=2, H=2, g=3, d=7, S=50, W=5, P=6)
+    m, l, o, n = core.row_stats(pb)
+    g = pb.Hq // pb.H
+    r = 0
+    for li in range(pb.M):
+        for h in range(pb.Hq):
+            for w in range(pb.W):
+                vis = pb.pos <= pb.qpos[w]
+                s = pb.scale * (pb.K[li, h // g][vis] @ pb.Q[li, h, w])
+                mm = s.max()
+                e = np.exp(s - mm)
+                assert n[r] == vis.sum()
+                assert _close(m[r], mm, 1e-13) and _close(l[r], e.sum(), 1e-12)
+                assert np.allclose(o[r], (e[:, None] * pb.V[li, h // g][vis]).sum(axis=0) / e.sum(),
+                                   rtol=1e-11, atol=1e-14)
+                r += 1
+    assert r == len(m)
+
+
 def test_invariants():
     rng = np.random.default_rng(11)
     pb = _random_problem(rng, M=2, H=2, g=2, d=8, S=60, W=5, P=10)
