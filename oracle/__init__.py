@@ -9,7 +9,9 @@ Contents
   core   fp64 page/set deletion effects (explicit deletion and Eq. 6 closed
          form, in C), row statistics, the greedy joint test, lifecycle
          classification (Eq. 9-10), pending protection and retained-index
-         selection (Eq. 12-13), and the compaction gather (Eq. 4).
+         selection (Eq. 12-13), the compaction gather (Eq. 4), and a
+         per-token window-attention fill score (a reading: the paper
+         defines no fill score).
   brute  an independent pure-Python brute force over every page subset for
          tiny problems, used to pin ``core``.
 
@@ -31,6 +33,7 @@ from .core import (  # noqa: F401
     row_stats,
     select_indices,
     set_effect,
+    token_scores,
     STATE_NONE,
     STATE_CANDIDATE,
     STATE_DORMANT,

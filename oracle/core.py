@@ -155,6 +155,35 @@ def row_stats(pb: Problem, nthreads=None):
     return m, l, o, n
 
 
+def token_scores(pb: Problem) -> np.ndarray:
+    """Per-token fill score (the reading taken for the budget fill of Eq. 13,
+    which the paper leaves open; a window-attention score in the spirit of
+    SnapKV, which the paper cites for its probe windows): token i scores
+    the largest attention weight a_{p,i} = exp(s_{p,i} - m_p) / l_p it gets
+    from any window position p of any query head of a selected layer, and 0
+    when no query sees it.  Written from the softmax row by row in numpy.
+    Parity unpinned against the paper, which defines no fill score; pinned
+    against the mathematics (uniform attention, invariants, the C row
+    statistics)."""
+    score = np.zeros(pb.S)
+    g = pb.Hq // pb.H
+    on = pb.layers_on()
+    for li in range(pb.M):
+        if not on[li]:
+            continue
+        for h in range(pb.Hq):
+            Kh = pb.K[li, h // g]
+            for w in range(pb.W):
+                vis = pb.pos <= pb.qpos[w]
+                if not vis.any():
+                    continue
+                s_ = pb.scale * (Kh[vis] @ pb.Q[li, h, w])
+                e = np.exp(s_ - s_.max())
+                idx = np.flatnonzero(vis)
+                score[idx] = np.maximum(score[idx], e / e.sum())
+    return score
+
+
 def _drop_mask(pb: Problem, pages) -> np.ndarray:
     drop = np.zeros(pb.S, np.uint8)
     for E in pages:

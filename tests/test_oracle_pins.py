@@ -198,6 +198,63 @@ def test_row_stats_textbook():
     assert r == len(m)
 
 
+def test_token_scores_uniform_attention():
+    """K = 0: a window position that sees n tokens gives each of them 1/n,
+    so a token's score is 1 / (the fewest tokens seen by a position that
+    sees it); with the probe positions ascending that is the first one at or
+    after the token."""
+    rng = np.random.default_rng(23)
+    pb = _random_problem(rng, M=1, H=1, g=2, d=4, S=40, W=5, P=4)
+    pb0 = core.Problem(np.zeros_like(pb.K), pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len)
+    sc = core.token_scores(pb0)
+    for i in range(pb0.S):
+        seen_by = [w for w in range(pb0.W) if pb0.pos[i] <= pb0.qpos[w]]
+        want = 0.0 if not seen_by else 1.0 / (pb0.pos <= pb0.qpos[seen_by[0]]).sum()
+        assert _close(sc[i], want, 1e-14), i
+
+
+def test_token_scores_invariants():
+    rng = np.random.default_rng(29)
+    pb = _random_problem(rng, M=2, H=2, g=2, d=6, S=60, W=5, P=6)
+    sc = core.token_scores(pb)
+    unseen = pb.pos > pb.qpos.max()
+    assert (sc[unseen] == 0).all() and (sc[~unseen] > 0).all() and sc.max() <= 1.0
+    # values do not enter; K -> cK with scale -> scale / c changes nothing
+    pbv = core.Problem(pb.K, -3.0 * pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len)
+    assert np.array_equal(core.token_scores(pbv), sc)
+    pbk = core.Problem(2.0 * pb.K, pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len, scale=pb.scale / 2.0)
+    assert np.allclose(core.token_scores(pbk), sc, rtol=1e-12)
+    # one layer, one head, one position: the weights of a softmax sum to 1
+    one = core.Problem(pb.K[:1, :1], pb.V[:1, :1], pb.pos, pb.Q[:1, :1, -1:], pb.qpos[-1:], pb.page_start,
+                       pb.page_len)
+    assert _close(core.token_scores(one).sum(), 1.0, 1e-12)
+    # a layer mask leaves the max over the selected layers
+    pbl = core.Problem(pb.K, pb.V, pb.pos, pb.Q, pb.qpos, pb.page_start, pb.page_len,
+                       layer_mask=np.array([0, 1], np.uint8))
+    only1 = core.Problem(pb.K[1:], pb.V[1:], pb.pos, pb.Q[1:], pb.qpos, pb.page_start, pb.page_len)
+    assert np.array_equal(core.token_scores(pbl), core.token_scores(only1))
+
+
+def test_token_scores_match_row_stats():
+    """The same weights from the C oracle's row statistics (m, l):
+    a_{p,i} = exp(s_{p,i} - m_p) / l_p, maximised over the rows."""
+    rng = np.random.default_rng(31)
+    pb = _random_problem(rng, M=2, H=2, g=3, d=5, S=45, W=4, P=5)
+    m, l, _, _ = core.row_stats(pb)
+    g = pb.Hq // pb.H
+    want = np.zeros(pb.S)
+    r = 0
+    for li in range(pb.M):
+        for h in range(pb.Hq):
+            for w in range(pb.W):
+                vis = pb.pos <= pb.qpos[w]
+                s_ = pb.scale * (pb.K[li, h // g] @ pb.Q[li, h, w])
+                a = np.where(vis, np.exp(s_ - m[r]) / l[r], 0.0)
+                want = np.maximum(want, a)
+                r += 1
+    assert np.allclose(core.token_scores(pb), want, rtol=1e-12, atol=1e-15)
+
+
 def test_invariants():
     rng = np.random.default_rng(11)
     pb = _random_problem(rng, M=2, H=2, g=2, d=8, S=60, W=5, P=10)
