@@ -6,8 +6,8 @@
  * deleting each event page of an agent's KV cache changes the attention
  * outputs of a probe window of queries, once before a tool-call commit and
  * once after the returned observation is in the cache (Section 3.2,
- * Eq. 5-8); classifies the pages' lifecycle states (Section 3.3, Eq. 9-10);
- * runs the greedy joint test on the completion candidates (Section 3.4,
+ * Eq. 5-8); classifies the pages' lifecycle states (Section 3.2, Eq. 9-10);
+ * runs the greedy joint test on the completion candidates (Section 3.3,
  * Eq. 11); and at a compression checkpoint keeps a bounded set of pending
  * pages and fills the budget, applying one index set to keys, values and
  * absolute positions (Eq. 4, 12, 13).
@@ -207,8 +207,8 @@ commitkv_status commitkv_page_effects_from_stats(const commitkv_shape *shape, in
                                                  size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Lifecycle classification, Section 3.3, Eq. 9-10, and the candidate order
- * of Section 3.4.
+ * Lifecycle classification, Section 3.2, Eq. 9-10, and the candidate order
+ * of Section 3.3.
  *
  * E_c = pages with eligible[E] != 0.  P-(E), P+(E) = #{F in E_c : R(F) <
  * R(E)} / |E_c| (ties share the lower rank).  H = (R >= tau_use and
@@ -264,7 +264,7 @@ commitkv_status commitkv_classify_variant(int32_t n_traj, const int32_t *P, cons
                                           cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Greedy joint test, Section 3.4, Eq. 11 and the inner loop of Algorithm 1.
+ * Greedy joint test, Section 3.3, Eq. 11 and the inner loop of Algorithm 1.
  *
  * Per trajectory, with A = {} and the candidates in the order given:
  * accept cand[j] iff R+(A u {cand[j]}) <= tau_joint, where R+(A) is Eq. 6-7
@@ -292,7 +292,7 @@ commitkv_status commitkv_joint_test(const commitkv_shape *shape, int32_t n_traj,
                                     cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Compression checkpoint, Section 3.4, Eq. 12-13, applied by Eq. 4.
+ * Compression checkpoint, Section 3.3, Eq. 12-13, applied by Eq. 4.
  *
  * Per trajectory: tokens of retired pages (D_c) are excluded.  Pending
  * pages that are not retired are ordered by decreasing pending_priority
@@ -330,7 +330,7 @@ commitkv_status commitkv_compact(const commitkv_shape *shape, int32_t n_traj,
                                  void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
- * Compression checkpoint in place, Section 3.4, Eq. 12-13 and Eq. 4.
+ * Compression checkpoint in place, Section 3.3, Eq. 12-13 and Eq. 4.
  *
  * The selection of commitkv_compact (same arguments and rules, same idx_out
  * and n_idx_out), with the gather done inside the cache: K and V row I_j of
@@ -378,7 +378,10 @@ commitkv_status commitkv_compact_in_place(const commitkv_shape *shape, int32_t n
  *     array's device address (cudaGetSymbolAddress, which may also load the
  *     library's device code on that device).  Make that first call before
  *     any stream capture on that device.  A failed look-up returns
- *     COMMITKV_ERR_CUDA.
+ *     COMMITKV_ERR_CUDA.  The address is kept for the life of the process:
+ *     it belongs to the device's primary context, so a process that
+ *     destroys that context (cudaDeviceReset) must not call this entry
+ *     point on that device afterwards.
  *   - Sharing: every call on a device uses the same array.  Calls whose
  *     work can overlap on the GPU (different streams, different host
  *     threads) race on it and give wrong results; serialise them, for

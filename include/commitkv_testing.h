@@ -2,7 +2,7 @@
  * commitkv_testing.h — test support of libcommitkv.so (not part of the hot
  * path).
  *
- * The greedy joint test (Section 3.4, Eq. 11) runs as one cooperative kernel
+ * The greedy joint test (Section 3.3, Eq. 11) runs as one cooperative kernel
  * whose blocks meet at a grid barrier once per candidate; every wait at that
  * barrier is bounded (about one second), after which the kernel records
  * COMMITKV_ERR_TIMEOUT in the workspace status word and returns, leaving the

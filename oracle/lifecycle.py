@@ -7,7 +7,7 @@ commits, in the order of Algorithm 1, with plain Python bookkeeping:
   pre_commit   commit c_t: the pages of every completed tool-call or
                observation event are measurable (E_{c_t}); R- over the
                pre-commit window (Eq. 5-8).  They wait for their post-commit
-               measurement (pending, Section 3.4 "Protecting incomplete
+               measurement (pending, Section 3.3 "Protecting incomplete
                transitions").
   checkpoint   Eq. 12-13 and Eq. 4: the retired pages D_c are excluded, at
                most B_N = floor(eta B) tokens and at most cap pages of the

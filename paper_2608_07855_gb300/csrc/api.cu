@@ -12,22 +12,6 @@ namespace ckv {
 int simt_rows_per_block();
 int simt_pages_per_block();
 int compact_max_pending();
-}  // namespace ckv
-
-using namespace ckv;
-
-namespace {
-
-constexpr size_t kAlign = 256;
-
-size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
-
-int layers_selected(const commitkv_shape *s, const uint8_t *mask, uint8_t *ids) {
-  int n = 0;
-  for (int l = 0; l < s->layers; ++l)
-    if (!mask || mask[l]) ids[n++] = (uint8_t)l;
-  return n;
-}
 
 commitkv_status check_shape(const commitkv_shape *s) {
   if (!s) return COMMITKV_ERR_INVALID_ARG;
@@ -55,6 +39,48 @@ commitkv_status check_trajs(const commitkv_shape *s, int n_traj, const commitkv_
     if ((int64_t)(s->q_heads / s->kv_heads) * x.W > (1 << 24)) return COMMITKV_ERR_INVALID_ARG;
   }
   return COMMITKV_OK;
+}
+
+// Host-side checks of the compression checkpoint's arguments, shared by
+// commitkv_compact, commitkv_compact_in_place and commitkv_compact_noalloc.
+commitkv_status check_compact_args(const commitkv_shape *s, int32_t n_traj, const commitkv_traj *tr,
+                                   const uint8_t *const *retired, const int32_t *const *pending,
+                                   const int32_t *n_pending, const float *const *pending_priority,
+                                   const float *const *fill_score, int32_t budget_B,
+                                   int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                   int32_t *const *idx_out, const int32_t *n_idx_out) {
+  commitkv_status st = check_shape(s);
+  if (st) return st;
+  if ((st = check_trajs(s, n_traj, tr, false))) return st;
+  if (budget_B < 0 || pending_tokens_BN < 0 || pending_tokens_BN > budget_B || pending_cap_pages < 0)
+    return COMMITKV_ERR_INVALID_ARG;
+  if (!retired || !n_pending || !fill_score || !idx_out || !n_idx_out) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t) {
+    if (n_pending[t] < 0 || n_pending[t] > compact_max_pending()) return COMMITKV_ERR_INVALID_ARG;
+    if (n_pending[t] > 0 && (!pending || !pending[t] || !pending_priority || !pending_priority[t]))
+      return COMMITKV_ERR_INVALID_ARG;
+    if (tr[t].P > 0 && !retired[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (tr[t].S > 0 && !fill_score[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (budget_B > 0 && !idx_out[t]) return COMMITKV_ERR_INVALID_ARG;
+  }
+  return COMMITKV_OK;
+}
+
+}  // namespace ckv
+
+using namespace ckv;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+int layers_selected(const commitkv_shape *s, const uint8_t *mask, uint8_t *ids) {
+  int n = 0;
+  for (int l = 0; l < s->layers; ++l)
+    if (!mask || mask[l]) ids[n++] = (uint8_t)l;
+  return n;
 }
 
 TrajDev to_dev(const commitkv_traj &x) {
@@ -566,20 +592,10 @@ static commitkv_status compact_impl(const commitkv_shape *shape, int32_t n_traj,
                                     void *const *k_out, void *const *v_out, int32_t *const *pos_out,
                                     void *workspace, size_t workspace_bytes, cudaStream_t stream,
                                     bool in_place) {
-  commitkv_status st = check_shape(shape);
+  commitkv_status st = check_compact_args(shape, n_traj, cache, retired, pending, n_pending, pending_priority,
+                                          fill_score, budget_B, pending_tokens_BN, pending_cap_pages, idx_out,
+                                          n_idx_out);
   if (st) return st;
-  if ((st = check_trajs(shape, n_traj, cache, false))) return st;
-  if (budget_B < 0 || pending_tokens_BN < 0 || pending_tokens_BN > budget_B || pending_cap_pages < 0)
-    return COMMITKV_ERR_INVALID_ARG;
-  if (!retired || !n_pending || !fill_score || !idx_out || !n_idx_out) return COMMITKV_ERR_INVALID_ARG;
-  for (int t = 0; t < n_traj; ++t) {
-    if (n_pending[t] < 0 || n_pending[t] > compact_max_pending()) return COMMITKV_ERR_INVALID_ARG;
-    if (n_pending[t] > 0 && (!pending || !pending[t] || !pending_priority || !pending_priority[t]))
-      return COMMITKV_ERR_INVALID_ARG;
-    if (cache[t].P > 0 && !retired[t]) return COMMITKV_ERR_INVALID_ARG;
-    if (cache[t].S > 0 && !fill_score[t]) return COMMITKV_ERR_INVALID_ARG;
-    if (budget_B > 0 && !idx_out[t]) return COMMITKV_ERR_INVALID_ARG;
-  }
   if ((st = check_ws(workspace, workspace_bytes, kAlign + compact_bytes(n_traj, cache)))) return st;
   static thread_local CompactLaunch L;
   memset(&L, 0, sizeof L);

@@ -96,6 +96,17 @@ __device__ __forceinline__ float effect_value(int n_del, int n_vis, float S_del,
   return sqrtf(num2) / (rest * onorm);
 }
 
+// Host-side argument checks (api.cu), shared by every entry point that
+// takes these arguments so that they refuse the same inputs.
+commitkv_status check_shape(const commitkv_shape *s);
+commitkv_status check_trajs(const commitkv_shape *s, int n_traj, const commitkv_traj *tr, bool need_q);
+commitkv_status check_compact_args(const commitkv_shape *s, int32_t n_traj, const commitkv_traj *tr,
+                                   const uint8_t *const *retired, const int32_t *const *pending,
+                                   const int32_t *n_pending, const float *const *pending_priority,
+                                   const float *const *fill_score, int32_t budget_B,
+                                   int32_t pending_tokens_BN, int32_t pending_cap_pages,
+                                   int32_t *const *idx_out, const int32_t *n_idx_out);
+
 // Launch helpers implemented in the .cu files ------------------------------
 
 struct ScoreLaunch {

@@ -1,5 +1,5 @@
-// Lifecycle classification (Section 3.3, Eq. 9-10) and candidate ordering
-// (Section 3.4), in two kernels:
+// Lifecycle classification (Section 3.2, Eq. 9-10) and candidate ordering
+// (Section 3.3), in two kernels:
 //   state  one warp per page (32 pages per block, every trajectory): the
 //          percentile ranks of R- and R+ among the eligible pages are plain
 //          counting compares split over the lanes; the page's state and

@@ -1,4 +1,4 @@
-// Compression checkpoint (Section 3.4, Eq. 12-13) and the shared-index
+// Compression checkpoint (Section 3.3, Eq. 12-13) and the shared-index
 // gather of keys, values and absolute positions (Eq. 4).
 //
 // select  one block per trajectory: mark retired tokens, protect the
@@ -116,6 +116,16 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
     s_order[rank] = E;
   }
   __syncthreads();
+  // Every check above has run (NaN fill scores, page spans, pending ids,
+  // duplicates): a failed one ends the trajectory here, before any page span
+  // is used to index the class bytes or a duplicate leaves a rank unwritten.
+  if (s_bad) {
+    if (threadIdx.x == 0) {
+      record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, -5);
+      L.n_idx[t] = 0;
+    }
+    return;
+  }
   if (threadIdx.x == 0) {
     // live entries occupy ranks [0, n_live); take the longest prefix that
     // fits both the page cap and the token budget B_N (Eq. 12)
@@ -142,13 +152,6 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
     for (int i = tr.ps[E] + threadIdx.x; i < tr.ps[E] + tr.pl[E]; i += kThreads) cls[i] = 2;
   }
   __syncthreads();
-  if (s_bad) {
-    if (threadIdx.x == 0) {
-      record_error(hdr, COMMITKV_ERR_DEVICE_INPUT, -5);
-      L.n_idx[t] = 0;
-    }
-    return;
-  }
   // fill: other non-retired tokens by (score desc, index desc) within the room
   int rem_local = 0;
   for (int i = threadIdx.x; i < S; i += kThreads) rem_local += cls[i] == 0;

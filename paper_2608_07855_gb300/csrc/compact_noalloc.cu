@@ -20,10 +20,6 @@
 
 #include "ckv_internal.cuh"
 
-namespace ckv {
-int compact_max_pending();
-}  // namespace ckv
-
 using namespace ckv;
 
 namespace {
@@ -67,41 +63,6 @@ commitkv_status scratch_for_current_device(void **out) {
   return COMMITKV_OK;
 }
 
-// The same host-side checks as commitkv_compact.
-commitkv_status check_args(const commitkv_shape *s, int32_t n_traj, const commitkv_traj *tr,
-                           const uint8_t *const *retired, const int32_t *const *pending,
-                           const int32_t *n_pending, const float *const *pending_priority,
-                           const float *const *fill_score, int32_t budget_B,
-                           int32_t pending_tokens_BN, int32_t pending_cap_pages,
-                           int32_t *const *idx_out, const int32_t *n_idx_out) {
-  if (!s) return COMMITKV_ERR_INVALID_ARG;
-  if (s->layers < 1 || s->layers > kMaxLayers || s->kv_heads < 1 || s->q_heads < s->kv_heads ||
-      s->q_heads % s->kv_heads != 0 || s->head_dim < 1)
-    return COMMITKV_ERR_INVALID_ARG;
-  if (s->dtype != COMMITKV_F32 && s->dtype != COMMITKV_BF16) return COMMITKV_ERR_INVALID_ARG;
-  if (!(s->softmax_scale >= 0.0f) || isinf(s->softmax_scale)) return COMMITKV_ERR_INVALID_ARG;
-  if (s->head_dim != 64 && s->head_dim != 128) return COMMITKV_ERR_UNSUPPORTED;
-  if (n_traj < 1 || n_traj > kMaxTraj || !tr) return COMMITKV_ERR_INVALID_ARG;
-  if (budget_B < 0 || pending_tokens_BN < 0 || pending_tokens_BN > budget_B || pending_cap_pages < 0)
-    return COMMITKV_ERR_INVALID_ARG;
-  if (!retired || !n_pending || !fill_score || !idx_out || !n_idx_out) return COMMITKV_ERR_INVALID_ARG;
-  for (int t = 0; t < n_traj; ++t) {
-    const commitkv_traj &x = tr[t];
-    if (x.S < 0 || x.W < 0 || x.P < 0) return COMMITKV_ERR_INVALID_ARG;
-    if (x.S > 0 && (!x.k || !x.v || !x.pos)) return COMMITKV_ERR_INVALID_ARG;
-    if (x.P > 0 && (!x.page_start || !x.page_len)) return COMMITKV_ERR_INVALID_ARG;
-    if (x.stride_tok < s->head_dim || x.stride_head < 0 || x.stride_layer < 0)
-      return COMMITKV_ERR_INVALID_ARG;
-    if (n_pending[t] < 0 || n_pending[t] > compact_max_pending()) return COMMITKV_ERR_INVALID_ARG;
-    if (n_pending[t] > 0 && (!pending || !pending[t] || !pending_priority || !pending_priority[t]))
-      return COMMITKV_ERR_INVALID_ARG;
-    if (x.P > 0 && !retired[t]) return COMMITKV_ERR_INVALID_ARG;
-    if (x.S > 0 && !fill_score[t]) return COMMITKV_ERR_INVALID_ARG;
-    if (budget_B > 0 && !idx_out[t]) return COMMITKV_ERR_INVALID_ARG;
-  }
-  return COMMITKV_OK;
-}
-
 }  // namespace
 
 extern "C" commitkv_status commitkv_compact_noalloc(
@@ -111,9 +72,10 @@ extern "C" commitkv_status commitkv_compact_noalloc(
     int32_t pending_tokens_BN, int32_t pending_cap_pages, int32_t *const *idx_out,
     int32_t *n_idx_out, void *const *k_out, void *const *v_out, int32_t *const *pos_out,
     int32_t *status_out, cudaStream_t stream) {
-  commitkv_status st = check_args(shape, n_traj, cache, retired, pending, n_pending,
-                                  pending_priority, fill_score, budget_B, pending_tokens_BN,
-                                  pending_cap_pages, idx_out, n_idx_out);
+  // the host-side checks of commitkv_compact, shared with it
+  commitkv_status st = check_compact_args(shape, n_traj, cache, retired, pending, n_pending,
+                                          pending_priority, fill_score, budget_B, pending_tokens_BN,
+                                          pending_cap_pages, idx_out, n_idx_out);
   if (st) return st;
   // Sizes beyond the fixed array are refused before anything is launched.
   size_t need = kAlign;

@@ -1,4 +1,4 @@
-// Greedy joint test (Section 3.4, Eq. 11; inner loop of Algorithm 1) on the
+// Greedy joint test (Section 3.3, Eq. 11; inner loop of Algorithm 1) on the
 // CUDA cores: the path for fp32 caches, head_dim 64 and rows that the
 // tensor-core kernel (joint_tc.cu) cannot stage; launch_joint chooses.
 //

@@ -1,4 +1,4 @@
-// Pieces of the greedy joint test (Section 3.4, Eq. 11) shared by its two
+// Pieces of the greedy joint test (Section 3.3, Eq. 11) shared by its two
 // kernels (CUDA-core and tensor-core): the round structure, the grid
 // barrier of the cooperative launch and the replay of a round's decisions.
 //

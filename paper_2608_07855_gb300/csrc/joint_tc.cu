@@ -1,4 +1,4 @@
-// Greedy joint test (Section 3.4, Eq. 11) on the 5th-generation tensor
+// Greedy joint test (Section 3.3, Eq. 11) on the 5th-generation tensor
 // cores: bf16 K/V/Q, head_dim 128, fp32 accumulation in tensor memory.
 //
 // One cooperative persistent kernel, one CTA of 256 threads per SM.  A

@@ -566,6 +566,37 @@ def test_device_input_errors_are_reported():
     assert b.status() == ck.COMMITKV_OK
 
 
+def test_compact_pending_span_out_of_range():
+    """A pending page whose span starts just past the cache (S + 1, inside
+    the 256-byte padding of the trajectory's token-class bytes in the
+    workspace) is reported as a device input error with |I| = 0, and the
+    selection writes no class byte outside [0, S): the padding byte keeps
+    the value it had before the call."""
+    r = get_run("small", 0)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    S = dev.tr.S_post
+    assert S % 256 != 0 and S + 1 < (S + 255) // 256 * 256  # the span's start lies in the padding
+    p = int(dev.tr.pending[0])
+    ps, pl = dev.page_start.clone(), dev.page_len.clone()
+    ps[p], pl[p] = S + 1, 1
+    t = ck.TrajTensors(dev.K, dev.V, dev.pos, dev.Q_post, dev.qpos_post, ps, pl)
+    retired = torch.zeros(dev.P_post, dtype=torch.uint8, device="cuda")
+    # token classes of the first trajectory start 256 bytes into the workspace
+    sentinel = 0x77
+    b.ws[256 + S + 1] = sentinel
+    b.n_idx.fill_(-1)
+    ck.commitkv_compact(b.shape, [t], [retired], [dev.pending], b.R_post, [dev.fill], cfg.B, cfg.B_N,
+                        cfg.pending_cap, b.idx, b.n_idx, workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_ERR_DEVICE_INPUT
+    assert int(b.n_idx[0]) == 0
+    assert int(b.ws[256 + S + 1]) == sentinel
+    # the context is still usable
+    b.score_post()
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+
+
 def test_bounded_wait_times_out():
     """A grid barrier that can never fill ends by its time limit with
     COMMITKV_ERR_TIMEOUT, and the context stays usable."""

@@ -40,13 +40,19 @@ def _fake_traj(S):
     return t
 
 
-def _call_raw(trajs, B=16):
+def _call_raw(trajs, B=16, shape=None, workspace_entry=False):
+    """commitkv_compact_noalloc (or, with workspace_entry, commitkv_compact
+    with a fake workspace) on descriptors that only the host checks read."""
     lib = ck.load_library()
     n = len(trajs)
     arr = (ck.Traj * n)(*trajs)
-    shape = ck.make_shape(1, 1, 1, 64, ck.COMMITKV_F32)
+    shape = shape or ck.make_shape(1, 1, 1, 64, ck.COMMITKV_F32)
     ptrs = (ctypes.c_void_p * n)(*([256] * n))
     npend = (ctypes.c_int32 * n)()
+    if workspace_entry:
+        return lib.commitkv_compact(ctypes.byref(shape), n, arr, ptrs, None,
+                                    ctypes.cast(npend, ctypes.c_void_p), None, ptrs, B, 0, 0,
+                                    ptrs, 256, None, None, None, 256, 1 << 20, None)
     return lib.commitkv_compact_noalloc(ctypes.byref(shape), n, arr, ptrs, None,
                                         ctypes.cast(npend, ctypes.c_void_p), None, ptrs, B, 0, 0,
                                         ptrs, 256, None, None, None, None, None)
@@ -61,6 +67,24 @@ def test_sizes_beyond_scratch_are_refused():
     assert _call_raw([_fake_traj(SCRATCH_BYTES - 256 + 1)]) == ck.COMMITKV_ERR_WORKSPACE
     assert _call_raw([_fake_traj(SCRATCH_BYTES // 2)] * 2) == ck.COMMITKV_ERR_WORKSPACE
     assert _call_raw([_fake_traj(SCRATCH_BYTES)] * 3) == ck.COMMITKV_ERR_WORKSPACE
+
+
+def test_host_checks_match_workspace_entry_point():
+    """Both compaction entry points share one set of host-side checks: shapes
+    and descriptors that commitkv_compact refuses, the no-alloc call refuses
+    with the same code, before any CUDA call."""
+    over_heads = ck.make_shape(2, 1, (1 << 19) + 1, 64, ck.COMMITKV_F32)  # layers * q_heads > 2^20
+    bad_dim = ck.make_shape(1, 1, 1, 96, ck.COMMITKV_F32)
+    bad_gqa = ck.make_shape(1, 2, 3, 64, ck.COMMITKV_F32)
+    small = _fake_traj(1024)
+    short = _fake_traj(1024)
+    short.stride_tok = 32  # below head_dim
+    cases = [(over_heads, [small], 16), (bad_dim, [small], 16), (bad_gqa, [small], 16),
+             (None, [short], 16), (None, [small], -1)]
+    for shape, trajs, B in cases:
+        want = _call_raw(trajs, B, shape, workspace_entry=True)
+        assert want in (ck.COMMITKV_ERR_INVALID_ARG, ck.COMMITKV_ERR_UNSUPPORTED)
+        assert _call_raw(trajs, B, shape) == want
 
 
 # ---------------------------------------------------------------------------
