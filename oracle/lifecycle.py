@@ -132,13 +132,14 @@ class OracleSession:
         Rm = np.asarray([self.R_pre.get(pid, 0.0) if eligible[i] else 0.0 for i, pid in enumerate(ids)])
         # later stages take fp32 effects, as the library's interface does
         Rm32, Rp32 = Rm.astype(np.float32), Rp.astype(np.float32)
-        _, cand = core.classify(Rm32, Rp32, eligible, **self.th, no_precommit=self.no_precommit,
-                                no_percentile=self.no_percentile)
+        state, cand = core.classify(Rm32, Rp32, eligible, **self.th, no_precommit=self.no_precommit,
+                                    no_percentile=self.no_percentile)
         cand = cand[:self.scan_cap]
         acc, step = core.greedy(pb, cand, self.tau_joint, "closed", stats=core.row_stats(pb))
         accepted = [ids[E] for E in cand if acc[E]]
         self.retired |= set(accepted)
         self.measured = []
-        out = dict(R_post=Rp, R_pre=Rm, cand=[ids[E] for E in cand], accepted=accepted, step_R=np.asarray(step))
+        out = dict(R_post=Rp, R_pre=Rm, cand=[ids[E] for E in cand], accepted=accepted, step_R=np.asarray(step),
+                   eligible=[pid for i, pid in enumerate(ids) if eligible[i]], state=np.asarray(state))
         self.log.append(("post", out))
         return out

@@ -66,3 +66,97 @@ def test_oracle_lifecycle_invariants():
             assert not (set(out["cand"]) & gone)
             n_acc += len(out["accepted"])
     assert n_ck >= 2 and n_acc >= 1, (n_ck, n_acc)
+
+
+def _hand():
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "lifecycle_hand.json")) as f:
+        return json.load(f)
+
+
+def _val(expr):
+    """A hand-derived closed form of the golden file: '0' or 'sqrt(a/b)'."""
+    from fractions import Fraction
+    if expr == "0":
+        return 0.0
+    assert expr.startswith("sqrt(") and expr.endswith(")")
+    return float(np.sqrt(float(Fraction(expr[5:-1]))))
+
+
+def _run_hand(g, scan_cap=None):
+    """Drives an OracleSession through the golden timeline; yields
+    (step, session, output) after every step."""
+    s = g["setup"]
+    o = OracleSession(s["M"], s["H"], s["Hq"], s["d"], s["G"], s["B"], s["eta"],
+                      scan_cap=s["scan_cap"] if scan_cap is None else scan_cap,
+                      protect_cap=s["protect_cap"], thresholds=s["thresholds"], tau_joint=s["tau_joint"])
+    vals = np.asarray(s["values"], np.float64)
+    events = [tuple(e) for e in s["events"]]
+    Q = np.ones((s["M"], s["Hq"], s["W"], s["d"]))  # K = 0: every score is 0 whatever Q is
+    for step in s["steps"]:
+        if step[0] == "append":
+            a, b = step[1], step[2]
+            n = b - a
+            K = np.zeros((s["M"], s["H"], n, s["d"]))
+            V = np.broadcast_to(vals[a:b], (s["M"], s["H"], n, s["d"])).copy()
+            o.append(K, V, np.arange(a, b), [e for e in events if e[0] in ("call", "obs") and a <= e[1]
+                                              and e[1] + e[2] <= b])
+            continue
+        if step[0] == "pre":
+            out = o.pre_commit(Q, [step[1]])
+        elif step[0] == "checkpoint":
+            out = o.checkpoint(s["fill"]) if o.pos.shape[0] > s["B"] else None
+        else:
+            out = o.post_commit(Q, [step[1]])
+        yield step[0], o, out
+
+
+def test_hand_worked_timeline():
+    """Two commits on a five-page cache whose effects are exact closed forms
+    (tests/golden/lifecycle_hand.json): E_c at each post-commit (measured at
+    the latest pre-commit, not retired, the new observation excluded), the
+    pending set and its protection, the page spans after a checkpoint that
+    keeps part of a page, D_c growing at an acceptance and shrinking when
+    its page is compacted away, and a joint-test rejection."""
+    g = _hand()
+    exp = iter(g["expected"])
+    for kind, o, out in _run_hand(g):
+        e = next(exp)
+        assert e["step"] == kind
+        if kind == "pre":
+            assert o.page_ids() == e["page_ids"]
+            np.testing.assert_allclose(out, [_val(x) for x in e["R"]], rtol=1e-12, atol=1e-14)
+            assert sorted(o.measured) == e["measured"]
+        elif kind == "checkpoint":
+            assert (out is not None) == e["taken"]
+            if e["taken"]:
+                assert out.tolist() == e["I"]
+                assert o.pos.tolist() == e["pos"]
+                assert o.pages == e["pages"]
+                assert sorted(o.retired) == e["retired"]
+        else:
+            assert o.page_ids() == e["page_ids"]
+            np.testing.assert_allclose(out["R_post"], [_val(x) for x in e["R_post"]], rtol=1e-12, atol=1e-14)
+            assert out["eligible"] == e["eligible"]
+            assert out["state"].tolist() == e["state"]
+            assert out["cand"] == e["cand"] and out["accepted"] == e["accepted"]
+            np.testing.assert_allclose(out["step_R"], [_val(x) for x in e["step_R"]], rtol=1e-12, atol=1e-14)
+            assert sorted(o.retired) == e["retired"]
+    assert next(exp, None) is None
+
+
+def test_hand_worked_timeline_scan_cap():
+    """The ordered candidate list is cut to scan_cap pages (the paper scans
+    at most 64 per commit): with a cap of 0 commit 1 accepts nothing."""
+    g = _hand()
+    want = g["scan_cap_zero"]
+    posts = 0
+    for kind, o, out in _run_hand(g, scan_cap=0):
+        if kind == "post":
+            posts += 1
+            if posts == want["commit"]:
+                assert out["cand"] == want["cand"] and out["accepted"] == want["accepted"]
+                assert not o.retired
+                return
+    raise AssertionError("no post-commit step")
