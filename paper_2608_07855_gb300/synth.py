@@ -200,23 +200,23 @@ CONFIGS = {
     # 2. Qwen3-8B shape, 16K + 2K
     "qwen3_8b_16k": Config("qwen3_8b_16k", M=36, H=8, Hq=32, d=128, dtype="bf16", L_pre=16384,
                            L_obs=2048, W=32, G=32, B=4096, pending_cap=16, planted_frac=0.2,
-                           outlier_channels=4, plant="shared", alpha=8.0, beta=(5.0, 8.0),
+                           outlier_channels=4, plant="shared", alpha=12.0, beta=(8.0, 12.0),
                            gamma=8.0, nu=6.0),
     # 3. Qwen3-8B shape, 32K + 4K (headline)
     "qwen3_8b_32k": Config("qwen3_8b_32k", M=36, H=8, Hq=32, d=128, dtype="bf16", L_pre=32768,
                            L_obs=4096, W=32, G=32, B=8192, pending_cap=32, planted_frac=0.2,
-                           outlier_channels=4, plant="shared", alpha=8.0, beta=(5.0, 8.0),
+                           outlier_channels=4, plant="shared", alpha=12.0, beta=(8.0, 12.0),
                            gamma=8.0, nu=6.0),
     # 4. 16 ragged trajectories, Qwen3-8B shape
     "ragged16": Config("ragged16", M=36, H=8, Hq=32, d=128, dtype="bf16", L_pre=0, L_obs=0, W=32,
                        G=32, B=8192, pending_cap=16, planted_frac=0.2, outlier_channels=4,
-                       plant="shared", alpha=8.0, beta=(5.0, 8.0), gamma=8.0, nu=6.0, n_traj=16,
+                       plant="shared", alpha=12.0, beta=(8.0, 12.0), gamma=8.0, nu=6.0, n_traj=16,
                        ctx_range=(4096, 32768), obs_range=(256, 4096), turns_range=(4, 24)),
     # 5. Qwen3-32B shape, 128K + 8K
     "qwen3_32b_128k": Config("qwen3_32b_128k", M=64, H=8, Hq=64, d=128, dtype="bf16",
                              L_pre=131072, L_obs=8192, W=64, G=64, B=16384, pending_cap=16,
-                             planted_frac=0.05, outlier_channels=4, plant="shared", alpha=8.0,
-                             beta=(5.0, 8.0), gamma=8.0, nu=6.0),
+                             planted_frac=0.05, outlier_channels=4, plant="shared", alpha=12.0,
+                             beta=(8.0, 12.0), gamma=8.0, nu=6.0),
 }
 
 
@@ -280,7 +280,8 @@ class Trajectory:
         return int(self.page_start.shape[0])
 
 
-_T_K, _T_V, _T_QPRE, _T_QPOST, _T_DIR, _T_FILL, _T_EVENTS, _T_PLANT, _T_OUTL, _T_PNOISE, _T_RAGGED, _T_VDIR = range(12)
+_T_K, _T_V, _T_QPRE, _T_QPOST, _T_DIR, _T_FILL, _T_EVENTS, _T_PLANT, _T_OUTL, _T_PNOISE, _T_RAGGED, _T_VDIR, \
+    _T_ROWS = range(13)
 
 
 def _stream(traj: int, tensor: int, layer: int = 0, head: int = 0) -> int:
@@ -463,8 +464,13 @@ def _plant_shared(tr, l, kvh, Qpre, Qpost, tok, page_of_tok, beta_page, row_page
     every post-window query.  The group's queries get a common direction per
     window, q = n + gamma * c (c- for Q-, c+ for Q+, c+ orthogonal to c-);
     page j's keys are k = alpha * u_j - beta_j * c+ + sigma * n, with u_j the
-    unit pre-window query row_page[j] of the group with its c+ component
-    removed.  Post-window scores are then about -gamma * beta_j / sqrt(d)."""
+    unit pre-window query of a seeded row of the group (drawn per slice) with
+    its c+ and c- components removed.  The page then dominates the attention of its own
+    pre-window row (score about alpha) and of no other (without the c-
+    removal every planted page would score alpha * gamma / |q| against every
+    pre-window query, the planted pages would share the pre-window mass and
+    each one's own effect would stay small).  Post-window scores are about
+    -gamma * beta_j / sqrt(d)."""
     cfg = tr.cfg
     g, W, d = cfg.g, cfg.W, cfg.d
     dirs = normal(tr.seed, _stream(tr.index, _T_DIR, l, kvh), (2, d)).astype(np.float64)
@@ -474,8 +480,13 @@ def _plant_shared(tr, l, kvh, Qpre, Qpost, tok, page_of_tok, beta_page, row_page
     Qpost[l, kvh * g:(kvh + 1) * g] += np.float32(cfg.gamma) * cp.astype(np.float32)
     if len(tok) == 0:
         return
+    # the aligned pre-window row of each page is drawn anew for every
+    # (layer, KV head): pages that share a row in one slice split its mass,
+    # but each page has slices where it is alone in its row
+    drr = Draws(tr.seed, _stream(tr.index, _T_ROWS, l, kvh))
+    row_page = np.asarray([drr.randint(0, g * W - 1) for _ in beta_page], np.int64)
     qm = Qpre[l, kvh * g:(kvh + 1) * g].reshape(g * W, d).astype(np.float64)[row_page]
-    u = qm - (qm @ cp)[:, None] * cp[None, :]
+    u = qm - (qm @ cp)[:, None] * cp[None, :] - (qm @ cm)[:, None] * cm[None, :]
     u = u / np.maximum(np.linalg.norm(u, axis=1, keepdims=True), 1e-30)
     noise = normal(tr.seed, _stream(tr.index, _T_PNOISE, l, kvh), (len(tok), d)).astype(np.float64)
     k = cfg.alpha * u[page_of_tok] - beta_page[page_of_tok][:, None] * cp[None, :] + cfg.sigma * noise

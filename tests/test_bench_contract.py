@@ -46,3 +46,39 @@ def test_peaks_are_the_measured_ones():
         m = json.load(f)
     assert kind == "measured"
     assert peaks["hbm_gbs"] == m["hbm_gbs"] and peaks["bf16_tflops_sustained"] == m["bf16_tflops_sustained"]
+
+
+def test_reference_arm_reports_the_same_config_keys():
+    """The reference arm's line describes the workload with the same keys
+    and values as ours, and its CPU baseline names the host CPU model."""
+    args = types.SimpleNamespace(config="tiny", layers=0, seed=0, steps=1, warmup=0,
+                                 cpu_sample_seconds=0.5)
+    res = bench.run_reference(args, 0, 1)
+    cfg = synth.CONFIGS["tiny"]
+    trs = [synth.make_trajectory(cfg, 0, traj=0, values=False)]
+    assert res["config"] == bench.config_dict(cfg, trs, 1)
+    assert res["impl"] == "reference" and res["cpu_baseline"]["cpu_model"]
+    assert isinstance(res["config"]["L_pre"], list) and "budget" in res["config"]
+
+
+def test_joint_report_counts():
+    """Candidates, acceptances, rounds of four and time per candidate of
+    the joint test, summed over the trajectories of a step."""
+    import numpy as np
+
+    class T:
+        def __init__(self, n):
+            self.n = n
+
+        def cpu(self):
+            return self
+
+        def tolist(self):
+            return self.n
+
+    acc = [np.array([1, 0, 1, 1, 0], np.uint8), np.array([0, 1, 0], np.uint8)]
+    buf = types.SimpleNamespace(n_cand=T([5, 2]), accepted=[a for a in acc],
+                                trajs=[types.SimpleNamespace(P_post=5), types.SimpleNamespace(P_post=3)])
+    r = bench.joint_report(buf, 0.7)
+    assert r["n_cand"] == 7 and r["accepted"] == 4 and r["rejected"] == 3
+    assert r["rounds"] == 2 and abs(r["us_per_candidate"] - 100.0) < 1e-9

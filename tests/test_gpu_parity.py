@@ -367,20 +367,39 @@ def test_full_step(name, seed):
     assert np.array_equal(st[idx][safe], o.state[idx][safe])
     assert safe.any()
     nc = int(b.n_cand[0])
-    if (st == o.state).all() and nc == len(o.cand) and np.array_equal(_np(b.cand[0])[:nc], o.cand):
-        stepR = _np(b.step_R[0])[:nc]
-        safe_s = safe_threshold_mask(o.step_R, cfg.tau_joint, r.tol)
-        upto = nc if safe_s.all() else int(np.argmin(safe_s))
-        _assert_close(stepR[:upto], o.step_R[:upto], r.tol, "step R")
-        if upto == nc:
-            assert np.array_equal(_np(b.accepted[0])[:dev.P_post], o.accepted)
-            n = int(b.n_idx[0])
-            # pending order depends on R+ of the observation pages; compare
-            # the index set when those priorities are separated
-            pr = o.R_post[dev.tr.pending]
-            srt = np.sort(pr)
-            if len(srt) < 2 or np.all(np.diff(srt) > 2 * r.tol * srt[1:]):
-                assert np.array_equal(_np(b.idx[0])[:n], o.I)
+    gpu_cand = _np(b.cand[0])[:nc]
+    # the GPU's candidates are the oracle classifier's on the GPU's own effects
+    g_state, g_cand = core.classify(_np(b.R_pre[0]).astype(np.float64), _np(b.R_post[0]).astype(np.float64),
+                                    dev.tr.eligible)
+    assert np.array_equal(st, g_state)
+    assert np.array_equal(gpu_cand, g_cand)
+    # joint test on that candidate list against the oracle's scan of the same
+    # list, up to the first step whose margin is within the tolerance
+    acc_o, step_o = core.greedy(o.post, gpu_cand, cfg.tau_joint, "closed", stats=o.stats)
+    stepR = _np(b.step_R[0])[:nc]
+    safe_s = safe_threshold_mask(step_o, cfg.tau_joint, r.tol)
+    upto = nc if safe_s.all() else int(np.argmin(safe_s))
+    _assert_close(stepR[:upto], step_o[:upto], r.tol, "step R")
+    acc = _np(b.accepted[0])[:dev.P_post]
+    for j in range(upto):
+        assert acc[gpu_cand[j]] == acc_o[gpu_cand[j]], j
+    for j in range(nc):
+        assert acc[gpu_cand[j]] == (stepR[j] <= cfg.tau_joint), j  # each decision follows its step value
+    assert not acc[np.setdiff1d(np.arange(dev.P_post), gpu_cand)].any()
+    # selection on the GPU's own decisions and priorities: bit-exact
+    n = int(b.n_idx[0])
+    R_post32 = _np(b.R_post[0])
+    I_g = core.select_indices(dev.tr.S_post, dev.tr.page_start, dev.tr.page_len, acc, dev.tr.pending,
+                              R_post32[dev.tr.pending].astype(np.float64), dev.tr.fill_score, cfg.B, cfg.B_N,
+                              cfg.pending_cap)
+    assert np.array_equal(_np(b.idx[0])[:n], I_g)
+    # and the oracle's own chain, where the GPU took the oracle's decisions
+    # and the pending priorities order alike
+    if np.array_equal(gpu_cand, o.cand) and np.array_equal(acc, o.accepted):
+        pr = o.R_post[dev.tr.pending]
+        srt = np.sort(pr)
+        if len(srt) < 2 or np.all(np.diff(srt) > 2 * r.tol * srt[1:]):
+            assert np.array_equal(_np(b.idx[0])[:n], o.I)
 
 
 def test_gapped_positions():
@@ -655,3 +674,41 @@ def test_many_zero_length_pages():
     Rw, _ = core.page_effects(post, "explicit")
     _assert_close(_np(buf.R_post[0]), Rw, 2e-2, "R+ with zero-length pages")
     assert (_np(buf.R_post[0])[np.asarray(pl) == 0] == 0).all()
+
+
+def test_qwen_shape_plain_normal_inputs():
+    """The Qwen3-8B shape (32 query / 8 KV heads, head_dim 128, bf16) with
+    Q, K, V ~ N(0, 1) as drawn (four key channels per (layer, KV head)
+    scaled by 8, no shared window direction, nothing planted), two layers of
+    a 4K + 512 cache: R-, R+ of every page and head, and the post-commit row
+    statistics, against the oracle's closed form (Eq. 6) over every slice."""
+    cfg = synth.small_config("qwen_n01", M=2, H=8, Hq=32, d=128, W=32, G=32, L_pre=4096, L_obs=512, B=1024,
+                             pending_cap=16, planted_frac=0.0, outlier_channels=4, plant="shared", gamma=0.0,
+                             alpha=0.0, beta=(0.0, 0.0), nu=0.0)
+    tr = synth.make_trajectory(cfg, 9)
+    assert len(tr.planted) == 0
+    dev = DeviceTrajectory.upload(tr)
+    b = StepBuffers(cfg, [dev])
+    headR_pre = torch.zeros(cfg.M, cfg.Hq, dev.P_pre, device="cuda")
+    headR_post = torch.zeros(cfg.M, cfg.Hq, dev.P_post, device="cuda")
+    R_pre = torch.zeros(dev.P_pre, device="cuda")
+    ck.commitkv_page_effects(b.shape, [dev.pre()], [R_pre], head_R_out=[headR_pre], workspace=b.ws)
+    ck.commitkv_page_effects(b.shape, [dev.post()], b.R_post, head_R_out=[headR_post], stats_out=b.stats,
+                             workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    from oracle_bridge import problems
+    pre, post = problems(tr)
+    Rm, Hm = core.page_effects(pre, "closed")
+    Rp, Hp = core.page_effects(post, "closed")
+    _assert_close(_np(R_pre), Rm, 2e-2, "R- (N(0,1) inputs)")
+    _assert_close(_np(b.R_post[0]), Rp, 2e-2, "R+ (N(0,1) inputs)")
+    _assert_close(_np(headR_pre), Hm, 2e-2, "R- per head (N(0,1) inputs)")
+    _assert_close(_np(headR_post), Hp, 2e-2, "R+ per head (N(0,1) inputs)")
+    m, l, o_vec, n = core.row_stats(post)
+    st = _np(b.stats[0]).reshape(-1, cfg.d + 4)
+    assert np.array_equal(st[:, 2].astype(np.int64), n)
+    _assert_close(st[:, 0], m, 1e-5, "row max")
+    _assert_close(st[:, 1], l, 1e-4, "row sum")
+    err = np.linalg.norm(st[:, 4:] - o_vec, axis=1) / np.maximum(np.linalg.norm(o_vec, axis=1), 1e-30)
+    assert err.max() <= 1e-4, err.max()
