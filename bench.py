@@ -70,6 +70,8 @@ def parse():
     ap.add_argument("--config", default="qwen3_8b_32k")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling cases)")
+    ap.add_argument("--kv-heads", type=int, default=0,
+                    help="override the KV head count, query heads scaled alike (profiling cases)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-sample-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -232,6 +234,9 @@ def config_of(args):
     cfg = synth.CONFIGS[args.config]
     if args.layers:
         cfg = dataclasses.replace(cfg, name=f"{cfg.name}_L{args.layers}", M=args.layers)
+    if getattr(args, "kv_heads", 0):
+        cfg = dataclasses.replace(cfg, name=f"{cfg.name}_H{args.kv_heads}", H=args.kv_heads,
+                                  Hq=cfg.g * args.kv_heads)
     return cfg
 
 

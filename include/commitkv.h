@@ -207,6 +207,39 @@ commitkv_status commitkv_page_effects_from_stats(const commitkv_shape *shape, in
                                                  size_t workspace_bytes, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Per-token fill scores for a compression checkpoint (Section 3.3, Eq. 13:
+ * the fill of the remaining budget).  The paper leaves the fill rule to an
+ * appendix it does not include; this is window attention in the spirit of
+ * SnapKV, whose probe windows the paper builds on:
+ *   scores_out[t][i] = max over selected layers l, query heads h and probe
+ *                      queries p with pos[i] <= q_pos[p] of
+ *                      exp(s_pi - m_p) / l_p,   s_pi = softmax_scale <q_p, k_i>,
+ * and 0 for a token that no probe query sees.  m_p and l_p are the row
+ * statistics of the same cache and window: pass the stats_out of a
+ * commitkv_page_effects call on this trajectory (a trajectory with P = 0
+ * pages gives the statistics alone).  Larger scores keep a token first.
+ *
+ *   shape, n_traj, trajs   as for commitkv_page_effects; k, pos, S, q,
+ *                          q_pos, W are read (v and the pages are not).
+ *   layer_mask   optional host [M] u8, the layers that take part (NULL: all).
+ *   stats        host array of n_traj device pointers, [M][Hq][W][d + 4]
+ *                fp32 as written by commitkv_page_effects (m, l used; the
+ *                rows of the selected layers are read).  Required when
+ *                S_t > 0 and W_t > 0.
+ *   scores_out   host array of n_traj device pointers, [S_t] fp32 each,
+ *                overwritten (required when S_t > 0).
+ *   workspace    at least 256 bytes, 256-byte aligned (the status word
+ *                only; any workspace of the other calls will do).
+ * Errors: INVALID_ARG for missing pointers or bad shapes, UNSUPPORTED for
+ * head_dim other than 64 and 128.  Tensor cores for bf16, head_dim 128 and
+ * 16-byte aligned rows (stats included); CUDA cores otherwise.
+ * -------------------------------------------------------------------- */
+commitkv_status commitkv_token_scores(const commitkv_shape *shape, int32_t n_traj, const commitkv_traj *trajs,
+                                      const uint8_t *layer_mask, const float *const *stats,
+                                      float *const *scores_out, void *workspace, size_t workspace_bytes,
+                                      cudaStream_t stream);
+
+/* ------------------------------------------------------------------------
  * Lifecycle classification, Section 3.2, Eq. 9-10, and the candidate order
  * of Section 3.3.
  *

@@ -98,9 +98,11 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.commitkv_compact_noalloc.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, vp, i32, i32,
                                              i32, vp, vp, vp, vp, vp, vp, vp]
     lib.commitkv_test_barrier_timeout.argtypes = [vp, sz, i32, vp]
+    lib.commitkv_token_scores.argtypes = [P(Shape), i32, P(Traj), vp, vp, vp, vp, sz, vp]
     for f in ("commitkv_workspace_init", "commitkv_workspace_status", "commitkv_page_effects",
-              "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_classify_variant", "commitkv_joint_test", "commitkv_compact",
-              "commitkv_compact_in_place", "commitkv_compact_noalloc", "commitkv_test_barrier_timeout"):
+              "commitkv_page_effects_from_stats", "commitkv_classify", "commitkv_classify_variant",
+              "commitkv_joint_test", "commitkv_compact", "commitkv_compact_in_place", "commitkv_compact_noalloc",
+              "commitkv_test_barrier_timeout", "commitkv_token_scores"):
         getattr(lib, f).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -281,6 +283,18 @@ def commitkv_page_effects_from_stats(shape: Shape, trajs, stats_in, R_out, head_
         ctypes.byref(shape), n, d, mptr, _ptr_array(stats_in, n), _ptr_array(R_out, n),
         _ptr_array(head_R_out, n), _ptr(workspace), workspace.numel(), _stream(stream))
     _check(rc, "commitkv_page_effects_from_stats")
+
+
+def commitkv_token_scores(shape: Shape, trajs, stats, scores_out, layer_mask=None, workspace=None, stream=None):
+    """Per-token fill scores (window attention with the given row stats)."""
+    n = len(trajs)
+    d = _descs(trajs)
+    _mbuf, mptr = _mask(layer_mask, shape.layers)
+    _require_cuda(*scores_out)
+    rc = load_library().commitkv_token_scores(
+        ctypes.byref(shape), n, d, mptr, _ptr_array(stats, n), _ptr_array(scores_out, n), _ptr(workspace),
+        workspace.numel(), _stream(stream))
+    _check(rc, "commitkv_token_scores")
 
 
 def commitkv_classify(P, R_pre, R_post, eligible, state_out, cand_out, n_cand_out, workspace,

@@ -9,6 +9,11 @@
 #include "score_tc.cuh"
 
 namespace ckv {
+namespace ts {
+cudaError_t launch_tc(const Batch &b, const float *const *stats, float *const *score, WsHeader *hdr,
+                      cudaStream_t s, int sm_count);
+cudaError_t launch_simt(const Batch &b, const float *const *stats, float *const *score, cudaStream_t s);
+}  // namespace ts
 int simt_rows_per_block();
 int simt_pages_per_block();
 int compact_max_pending();
@@ -179,15 +184,41 @@ int simt_chunk_bound(int S) {
   return c < 16 ? c : 16;
 }
 
-size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
-  size_t items = 0, slots = 0;
+// The single cooperative launch of both scoring passes is opt-in
+// (COMMITKV_FUSED=1): both passes are bound by their SMs' pipelines rather
+// than by HBM, so serving the page pass's re-reads from L2 does not make it
+// faster, and the fused launch measured slower than the separate launches.
+bool env_fused() {
+  const char *e = getenv("COMMITKV_FUSED");
+  return e && e[0] == '1';
+}
+
+// Flash-pass partial slots the tensor-core path may need for these caches or
+// smaller ones: one per item of the two-launch chunking, or the fused
+// launch's ring (at most kMaxFusedCtas x kPartialRing slots, and at most one
+// per item of its chunking: about kFusedItemsPerSlice items per slice).
+size_t tc_partial_slots(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
+  size_t items = 0, fused = 0;
   for (int t = 0; t < n_traj; ++t) {
     TcCounts c = tc_counts(s, tr[t], tc_chunk_len(1, &tr[t]));
     items += (size_t)s->layers * s->kv_heads * tc_chunk_bound(tr[t].S) * c.nrt;
+    fused += (size_t)s->layers * s->kv_heads * (tc::kFusedItemsPerSlice + 1 + c.nrt);
+  }
+  const size_t ring = (size_t)tc::kMaxFusedCtas * tc::kPartialRing;
+  if (fused > ring) fused = ring;
+  return items > fused ? items : fused;
+}
+
+size_t tc_score_bytes(const commitkv_shape *s, int n_traj, const commitkv_traj *tr) {
+  size_t slots = 0, slices = 0;
+  for (int t = 0; t < n_traj; ++t) {
+    TcCounts c = tc_counts(s, tr[t], tc_chunk_len(1, &tr[t]));
     slots += align_up((size_t)(tr[t].P + 1) * 4) + align_up((size_t)c.nbitem * 32) + kAlign +
              align_up(((size_t)cdiv(tr[t].S, 16) + tr[t].P) * 16);
+    slices += (size_t)s->layers * s->kv_heads;
   }
-  return align_up(items * tc::kPartsPerItem * tc::kRowsPerTile * 132 * 4) + slots;
+  return align_up(tc_partial_slots(s, n_traj, tr) * tc::kPartsPerItem * tc::kRowsPerTile * 132 * 4) +
+         align_up(slices * 2 * tc::kCounterStride * 4) + slots;
 }
 
 // Region sizes of each call (bytes after the 256-byte header).
@@ -375,14 +406,23 @@ commitkv_status page_effects_impl(const commitkv_shape *shape, int32_t n_traj, c
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return cuda_status(e);
+  const bool fused = !from_stats && env_fused();
   int CLt = tc_chunk_len(n_traj, trajs);
-  float *tc_partials = reinterpret_cast<float *>(base);
-  size_t items_all = 0;
-  for (int t = 0; t < n_traj; ++t) {
-    TcCounts c = tc_counts(shape, trajs[t], CLt);
-    items_all += (size_t)shape->layers * shape->kv_heads * tc_chunk_bound(trajs[t].S) * c.nrt;
+  if (fused) {
+    int smax = 0, nrt_max = 1;
+    for (int t = 0; t < n_traj; ++t) {
+      smax = trajs[t].S > smax ? trajs[t].S : smax;
+      const int nrt = cdiv(L.batch.g * trajs[t].W, tc::kRowsPerTile);
+      nrt_max = nrt > nrt_max ? nrt : nrt_max;
+    }
+    CLt = tc::fused_chunk_len(smax, nrt_max);
   }
-  char *slot_base = base + align_up(items_all * tc::kPartsPerItem * tc::kRowsPerTile * 132 * 4);
+  float *tc_partials = reinterpret_cast<float *>(base);
+  size_t slices_all = 0;
+  for (int t = 0; t < n_traj; ++t) slices_all += (size_t)shape->layers * shape->kv_heads;
+  char *cnt_base = base + align_up(tc_partial_slots(shape, n_traj, trajs) * tc::kPartsPerItem * tc::kRowsPerTile *
+                                   132 * 4);
+  char *slot_base = cnt_base + align_up(slices_all * 2 * tc::kCounterStride * 4);
   for (int b0 = 0; b0 < n_traj; b0 += tc::kMaxTc) {
     int nb = n_traj - b0 < tc::kMaxTc ? n_traj - b0 : tc::kMaxTc;
     memset(&T, 0, sizeof T);
@@ -397,6 +437,9 @@ commitkv_status page_effects_impl(const commitkv_shape *shape, int32_t n_traj, c
     T.from_stats = L.from_stats;
     T.scale_log2 = L.batch.scale_log2;
     T.partials = tc_partials;
+    T.fused = fused ? 1 : 0;
+    T.a_done = reinterpret_cast<uint32_t *>(cnt_base);
+    T.merged = T.a_done + slices_all * tc::kCounterStride;
     memcpy(T.layer_ids, L.batch.layer_ids, sizeof T.layer_ids);
     for (int i = 0; i < nb; ++i) {
       int t = b0 + i;
@@ -431,6 +474,7 @@ commitkv_status page_effects_impl(const commitkv_shape *shape, int32_t n_traj, c
       T.item_off_a[i + 1] = T.item_off_a[i] + ia;
       T.item_off_b[i + 1] = T.item_off_b[i] + ib;
       T.row_off[i + 1] = T.row_off[i] + (active ? nl * shape->kv_heads * L.batch.g * x.W : 0);
+      T.slice_off[i + 1] = T.slice_off[i] + (active ? nl * shape->kv_heads : 0);
       if (active && !tc::build_maps(T.maps[i], L.batch.t[t], shape->layers, shape->kv_heads, shape->q_heads))
         return COMMITKV_ERR_CUDA;
     }
@@ -459,6 +503,45 @@ commitkv_status commitkv_page_effects_from_stats(const commitkv_shape *shape, in
   if (!stats_in) return COMMITKV_ERR_INVALID_ARG;
   return page_effects_impl(shape, n_traj, trajs, layer_mask, stats_in, R_out, head_R_out, nullptr, workspace,
                            workspace_bytes, stream);
+}
+
+commitkv_status commitkv_token_scores(const commitkv_shape *shape, int32_t n_traj, const commitkv_traj *trajs,
+                                      const uint8_t *layer_mask, const float *const *stats,
+                                      float *const *scores_out, void *workspace, size_t workspace_bytes,
+                                      cudaStream_t stream) {
+  commitkv_status st = check_shape(shape);
+  if (st) return st;
+  if ((st = check_trajs(shape, n_traj, trajs, true))) return st;
+  if (!stats || !scores_out) return COMMITKV_ERR_INVALID_ARG;
+  for (int t = 0; t < n_traj; ++t) {
+    if (trajs[t].S > 0 && !scores_out[t]) return COMMITKV_ERR_INVALID_ARG;
+    if (trajs[t].S > 0 && trajs[t].W > 0 && !stats[t]) return COMMITKV_ERR_INVALID_ARG;
+  }
+  if ((st = check_ws(workspace, workspace_bytes, kAlign))) return st;
+  static thread_local Batch B;
+  fill_batch(B, shape, n_traj, trajs, layer_mask);
+  for (int t = 0; t < n_traj; ++t) {
+    if (trajs[t].S == 0) continue;
+    cudaError_t e = cudaMemsetAsync(scores_out[t], 0, (size_t)trajs[t].S * 4, stream);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  if (B.n_layers == 0) return COMMITKV_OK;
+  // tensor cores for bf16, head_dim 128 and 16-byte aligned rows
+  bool tc = shape->dtype == COMMITKV_BF16 && shape->head_dim == 128 && !env_force_simt();
+  for (int t = 0; t < n_traj && tc; ++t) {
+    const commitkv_traj &x = trajs[t];
+    if (x.S == 0 || x.W == 0) continue;
+    if (((uintptr_t)x.k | (uintptr_t)x.q | (uintptr_t)stats[t]) % 16) tc = false;
+    if ((x.stride_tok * 2) % 16 || (x.stride_head * 2) % 16 || (x.stride_layer * 2) % 16) tc = false;
+    if (x.stride_head == 0 || x.stride_layer == 0) tc = false;
+  }
+  WsHeader *hdr = static_cast<WsHeader *>(workspace);
+  if (!tc) return cuda_status(ts::launch_simt(B, stats, scores_out, stream));
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = ts::launch_tc(B, stats, scores_out, hdr, stream, sms);
+  return cuda_status(e);
 }
 
 commitkv_status commitkv_classify(int32_t n_traj, const int32_t *P, const float *const *R_pre,

@@ -21,6 +21,7 @@
 // Every mbarrier wait is bounded (1 s); on expiry the kernel records
 // COMMITKV_ERR_TIMEOUT and all warps leave their loops.
 #include <cudaTypedefs.h>
+#include <stdlib.h>
 
 #include "ckv_internal.cuh"
 #include "sm103.cuh"
@@ -42,6 +43,7 @@ constexpr int SLOTS = BT / SLOT;  // slots per pass-B tile
 constexpr int NFIFO = 16;         // page-sum FIFO depth (>= 2 x SLOTS)
 constexpr uint64_t kWait = 1000000000ull;
 constexpr float kLazy = 8.0f;     // rescale O when the max grows by > 2^8
+constexpr int kRing = kPartialRing;  // partial slots per flash CTA of the fused launch
 
 constexpr uint32_t kTileBytes = BT * D * 2;  // 32 KB (two 16 KB halves)
 constexpr uint32_t kHalf = kTileBytes / 2;
@@ -73,6 +75,82 @@ __device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int ks) {
   return smem_desc(smem_addr(tile) + ks * 2048, kHalf, 1024, kSwizzle128B);
 }
 
+// ============================================================== fused-launch plumbing
+// Partial slot of a flash-pass item.  The two-launch path keeps one slot per
+// item.  The fused launch keeps n_a * kRing slots: item i runs on CTA
+// i mod n_a and takes slot i mod (n_a * kRing), last used by the same CTA's
+// item i - n_a * kRing.
+template <bool FUSED>
+__device__ __forceinline__ float *part_ptr(const TcLaunch &L, int item, int h, int row) {
+  const int64_t slot = FUSED ? (int64_t)(item % (L.n_a * kRing)) : (int64_t)item;
+  return L.partials + ((slot * 2 + h) * BM + row) * (D + 4);
+}
+
+// Index of an item's (trajectory, layer, KV head) slice in the per-slice counters.
+template <class Item>
+__device__ __forceinline__ int slice_of(const TcLaunch &L, const Item &it) {
+  return (L.slice_off[it.t] + it.li * L.H + it.kvh) * kCounterStride;
+}
+__device__ __forceinline__ int items_per_slice(const TcLaunch &L, int t) { return L.t[t].nchunk * L.t[t].nrt; }
+
+// Called by all 32 lanes of a warp: waits until *p >= target (an acquire
+// load by every lane, so each lane's later reads see the writes released
+// with the counter).  Bounded: gives up on the CTA's or the launch's abort
+// flag, or after kWait, recording a timeout and raising both flags.
+__device__ __forceinline__ bool warp_poll_geq(const uint32_t *p, uint32_t target, volatile int *abort_flag,
+                                              WsHeader *hdr) {
+  uint64_t t0 = 0;
+  for (;;) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    if (__all_sync(0xffffffffu, v >= target)) return true;
+    const bool stop = *abort_flag || *reinterpret_cast<volatile int32_t *>(&hdr->abort);
+    const uint64_t now = now_ns();
+    if (t0 == 0) t0 = now;
+    const bool late = now - t0 > kWait;
+    if (__any_sync(0xffffffffu, stop || late)) {
+      if (late && (threadIdx.x & 31) == 0) {
+        *abort_flag = 1;
+        atomicExch(&hdr->abort, 1);
+        record_error(hdr, COMMITKV_ERR_TIMEOUT, 12);
+      }
+      return false;
+    }
+    __nanosleep(512);
+  }
+}
+
+// Partials of the fused launch are written once and read once soon after:
+// kept in L2 over the streaming K and V, dropped first after their read.
+__device__ __forceinline__ void st_keep(float *p, float4 v) {
+  asm volatile(
+      "{\n\t.reg .b64 pol;\n\tcreatepolicy.fractional.L2::evict_last.b64 pol, 1.0;\n\t"
+      "st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, pol;\n\t}" ::"l"(p),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+      : "memory");
+}
+__device__ __forceinline__ float4 ld_once(const float *p) {
+  float4 v;
+  asm volatile(
+      "{\n\t.reg .b64 pol;\n\tcreatepolicy.fractional.L2::evict_first.b64 pol, 1.0;\n\t"
+      "ld.global.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], pol;\n\t}"
+      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+      : "l"(p)
+      : "memory");
+  return v;
+}
+
+// Called by all 32 lanes after each wrote its part of a result: one
+// release increment of *p for the warp.
+__device__ __forceinline__ void signal_add(uint32_t *p, int lane) {
+  __threadfence();
+  __syncwarp();
+  if (lane == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p) : "memory");
+}
+
+template <bool FUSED>
+__device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int kvh, int row, int lane);
+
 // ============================================================== pass A
 // Two softmax warpgroups take alternate tiles of a chunk (global tile g goes
 // to warpgroup g & 1), each with its own S/P buffer, running max, sum and
@@ -86,8 +164,9 @@ struct SmemA {
   alignas(1024) uint8_t k[NKB][kTileBytes];
   alignas(1024) uint8_t v[NVB][kTileBytes];
   int pos[2][4][BT];  // per softmax warp: positions of the current tile
+  float4 pub[BM];     // fused launch: warpgroup 1's (reference max, sum, count, true max) of the item, per row
   uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2], s_empty[2], p_full[2],
-      pv_done[2], o_full[2], o_empty[2], drain, drain2;
+      pv_done[2], o_full[2], o_empty[2], drain, drain2, pub_full, pub_empty;
   uint32_t tmem;
   int abort_flag;
 };
@@ -133,8 +212,9 @@ __device__ __forceinline__ void issue_pv_step(uint32_t tm, uint32_t d_col, const
   mma_bf16_ts(tm + d_col, tm + p_col(b, ks, 1), bd, idesc, 1u);
 }
 
-__global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
-  extern __shared__ uint8_t smem_raw[];
+template <bool FUSED>
+__device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uint8_t *smem_raw, const int cta,
+                                           const int ncta) {
   SmemA &sm = *reinterpret_cast<SmemA *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_items = L.item_off_a[L.n_traj];
@@ -162,6 +242,8 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
     }
     mbar_init(&sm.drain, 1);
     mbar_init(&sm.drain2, 1);
+    mbar_init(&sm.pub_full, 4);   // warpgroup 1's warps: the item's state is published
+    mbar_init(&sm.pub_empty, 4);  // warpgroup 0's warps: the publication is consumed
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -177,14 +259,15 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
   // 2: softmax of the even and the odd tiles.  Register budget per thread:
   // 56 + 2 x 224 = the launch's 3 x 168.
   if (warp < 4) {
-    regs_dec<56>();  // warp 3 stays idle
+    if (FUSED) regs_dec<48>();
+    else regs_dec<56>();  // warp 3 stays idle
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
       if (lane == 0) {
         uint64_t pol = policy_evict_normal();
         uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
         bool stop = false;
-        for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x, ++n_local) {
+        for (int item = cta; item < n_items && !stop; item += ncta, ++n_local) {
           if (*abort_flag) break;
           ItemA a = decode_a(L, item);
           const TcTraj &tr = L.t[a.t];
@@ -238,7 +321,7 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
       uint32_t it = 0;
       int uses0 = 0, uses1 = 0;  // items in which O_0 / O_1 have been filled so far
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      for (int item = cta; item < n_items && ok; item += ncta) {
         ItemA a = decode_a(L, item);
         const TcTraj &tr = L.t[a.t];
         int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
@@ -282,7 +365,7 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
       if (lane == 0) {
         uint32_t it = 0, n_local = 0;
         bool ok = true;
-        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x, ++n_local) {
+        for (int item = cta; item < n_items && ok; item += ncta, ++n_local) {
           ItemA a = decode_a(L, item);
           const TcTraj &tr = L.t[a.t];
           int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
@@ -311,9 +394,10 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
         }
       }
     }
-  } else {
+  } else if (warp < 12) {
     // ------------------------------------------------------------ softmax (warps 4..11)
-    regs_inc<224>();
+    if (FUSED) regs_inc<208>();
+    else regs_inc<224>();
     const int hb = (warp - 4) >> 2;   // this warpgroup's tiles: g & 1 == hb
     const int wq = warp & 3;          // TMEM lane quarter of this warp
     const int row = wq * 32 + lane;   // probe row within the tile
@@ -322,8 +406,9 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
     int *posw = sm.pos[hb][wq];
     uint32_t it = 0;
     int uses = 0;  // items in which this warpgroup filled O_hb
+    uint32_t n_it = 0;  // items of this CTA seen so far (fused launch)
     bool ok = true;
-    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+    for (int item = cta; item < n_items && ok; item += ncta) {
       ItemA a = decode_a(L, item);
       const TcTraj &tr = L.t[a.t];
       int rows = L.g * tr.W;
@@ -334,7 +419,7 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
       int t0 = a.c * L.chunk_len, t1 = min(tr.S, t0 + L.chunk_len);
       int ntile = (t1 - t0 + BT - 1) / BT;
       const int j0 = (hb - (int)it) & 1;  // first tile of this warpgroup in the item
-      float *dst = L.partials + (((int64_t)item * 2 + hb) * BM + row) * (D + 4);
+      float *dst = part_ptr<FUSED>(L, item, hb, row);
       float m_used = -INFINITY, m_true = -INFINITY, lsum = 0.0f;
       int nvis = 0;
       for (int j = j0; j < ntile && ok; j += 2) {
@@ -446,6 +531,83 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
         if (lane == 0) mbar_arrive(&sm.p_full[b]);
       }
       if (!ok) break;
+      if (FUSED) {
+        // One partial per item: warpgroup 1 publishes its (reference max,
+        // sum, count, true max) and leaves its O in tensor memory; warpgroup
+        // 0 rescales both outputs to the larger reference max, writes the
+        // partial and hands both O accumulators back to the P V issuer.
+        const bool mine = j0 < ntile;  // this warpgroup filled its O in this item
+        if (hb == 1) {
+          if (n_it > 0 && !__all_sync(0xffffffffu, mbar_wait(&sm.pub_empty, (n_it - 1) & 1, kWait, abort_flag))) {
+            ok = false;
+            break;
+          }
+          if (mine && !__all_sync(0xffffffffu, mbar_wait(&sm.o_full[1], uses & 1, kWait, abort_flag))) {
+            ok = false;
+            break;
+          }
+          sm.pub[row] = make_float4(mine ? m_used : -INFINITY, lsum, (float)nvis, m_true);
+          if (mine) ++uses;
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.pub_full);
+        } else {
+          if (item >= L.n_a * kRing) {
+            // the partial slot was last used by this CTA's item kRing items
+            // back: its slice must be merged before the slot is overwritten
+            const ItemA pa = decode_a(L, item - L.n_a * kRing);
+            if (!warp_poll_geq(&L.merged[slice_of(L, pa)], 4u * items_per_slice(L, pa.t), abort_flag, hdr)) {
+              ok = false;
+              break;
+            }
+          }
+          if ((mine && !__all_sync(0xffffffffu, mbar_wait(&sm.o_full[0], uses & 1, kWait, abort_flag))) ||
+              !__all_sync(0xffffffffu, mbar_wait(&sm.pub_full, n_it & 1, kWait, abort_flag))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const float4 o1 = sm.pub[row];
+          const bool mine1 = (int)((1u - it) & 1u) < ntile;  // warpgroup 1 filled its O in this item
+          const bool theirs = mine1 && o1.x != -INFINITY;
+          const float m0 = mine ? m_used : -INFINITY;
+          const float mr = fmaxf(m0, theirs ? o1.x : -INFINITY);
+          const float f0 = m0 == -INFINITY ? 0.0f : exp2f(m0 - mr);
+          const float f1 = theirs ? exp2f(o1.x - mr) : 0.0f;
+#pragma unroll 1
+          for (int c0 = 0; c0 < D; c0 += 32) {
+            float x0[32], x1[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) x0[i] = x1[i] = 0.0f;
+            if (mine) tmem_ld32f(tm + lane_base + 2 * BT + c0, x0);
+            if (mine1) tmem_ld32f(tm + lane_base + 2 * BT + D + c0, x1);
+            tmem_wait_ld();
+            if (valid_row) {
+#pragma unroll
+              for (int i = 0; i < 32; i += 4)
+                st_keep(dst + 4 + c0 + i, make_float4(fmaf(x0[i], f0, theirs ? x1[i] * f1 : 0.0f),
+                                                      fmaf(x0[i + 1], f0, theirs ? x1[i + 1] * f1 : 0.0f),
+                                                      fmaf(x0[i + 2], f0, theirs ? x1[i + 2] * f1 : 0.0f),
+                                                      fmaf(x0[i + 3], f0, theirs ? x1[i + 3] * f1 : 0.0f)));
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            if (mine) mbar_arrive(&sm.o_empty[0]);
+            if (mine1) mbar_arrive(&sm.o_empty[1]);
+            mbar_arrive(&sm.pub_empty);
+          }
+          if (mine) ++uses;
+          // (reference max of l and O, sum, visible count, true max)
+          if (valid_row)
+            st_keep(dst, make_float4(mr, fmaf(lsum, f0, o1.y * f1), (float)nvis + o1.z, fmaxf(m_true, o1.w)));
+          signal_add(&L.a_done[slice_of(L, a)], lane);  // this warp's rows of the partial are written
+        }
+        ++n_it;
+        it += ntile;
+        continue;
+      }
       if (j0 < ntile) {
         // this warpgroup's O is complete after its last P V of the item
         if (!__all_sync(0xffffffffu, mbar_wait(&sm.o_full[hb], uses & 1, kWait, abort_flag))) {
@@ -476,55 +638,99 @@ __global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLa
       if (valid_row) *reinterpret_cast<float4 *>(dst) = make_float4(m_used, lsum, (float)nvis, m_true);
       it += ntile;
     }
+  } else if (FUSED) {
+    // ------------------------------------------------------------ merge (warps 12..15, fused launch only)
+    // For each item of this CTA, once every item of its slice has written
+    // its partials, the four warps merge this item's share of the slice's
+    // probe rows into the row statistics (m, l, n, o); the page-pass CTAs
+    // wait for all shares of a slice.  No tensor memory, no TMA.
+    regs_dec<48>();
+    const int w = warp - 12;
+    for (int item = cta; item < n_items; item += ncta) {
+      const ItemA a = decode_a(L, item);
+      const TcTraj &tr = L.t[a.t];
+      const int s = slice_of(L, a), nis = items_per_slice(L, a.t);
+      if (!warp_poll_geq(&L.a_done[s], 4u * nis, abort_flag, hdr)) break;
+      const int rows = L.g * tr.W, jin = a.c * tr.nrt + a.rt;
+      const int r0 = (int)((int64_t)jin * rows / nis), r1 = (int)((int64_t)(jin + 1) * rows / nis);
+      for (int row = r0 + w; row < r1; row += 4) merge_row<FUSED>(L, a.t, a.li, a.kvh, row, lane);
+      signal_add(&L.merged[s], lane);
+    }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tm, 512);
-  if (threadIdx.x == 0 && sm.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, 10);
+  if (threadIdx.x == 0 && sm.abort_flag) {
+    if (FUSED) atomicExch(&hdr->abort, 1);
+    record_error(hdr, COMMITKV_ERR_TIMEOUT, 10);
+  }
 }
 
+__global__ void __launch_bounds__(384, 1) pass_a_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  flash_body<false>(L, hdr, smem_raw, blockIdx.x, gridDim.x);
+}
+
+
 // ============================================================== combine
-// One warp per probe row of the selected layers.
-__global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaunch L) {
-  int gw = (blockIdx.x * 256 + threadIdx.x) / 32, lane = threadIdx.x % 32;
-  int total = L.row_off[L.n_traj];
-  if (gw >= total) return;
-  int t = traj_of(L.row_off, L.n_traj, gw);
+// Merges the 2 x nchunk partials of one probe row of a (trajectory, layer,
+// KV head) slice into its row stats (m, l, n, o): one warp, four channels
+// per lane.
+template <bool FUSED>
+__device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int kvh, int row, int lane) {
   const TcTraj &tr = L.t[t];
-  int local = gw - L.row_off[t];
-  int rows = L.g * tr.W;
-  int row = local % rows;
-  local /= rows;
-  int kvh = local % L.H, li = local / L.H;
-  int l = L.layer_ids[li];
-  int rt = row / BM, rl = row % BM;
-  // partial k = 2 c + h: chunk c, softmax warpgroup h
+  const int l = L.layer_ids[li];
+  const int rt = row / BM, rl = row % BM;
+  // fused launch: partial k = chunk k (one per item); otherwise partial
+  // k = 2 c + h: chunk c, softmax warpgroup h
   auto part = [&](int k) {
-    int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + (k >> 1)) * tr.nrt + rt;
-    return L.partials + (((int64_t)item * 2 + (k & 1)) * BM + rl) * (D + 4);
+    const int c = FUSED ? k : k >> 1;
+    const int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + c) * tr.nrt + rt;
+    return part_ptr<FUSED>(L, item, FUSED ? 0 : k & 1, rl);
   };
-  const int nparts = 2 * tr.nchunk;
-  float m = -INFINITY;  // true row max over the partials (base 2)
-  for (int k = 0; k < nparts; ++k) m = fmaxf(m, part(k)[3]);
+  const int nparts = FUSED ? tr.nchunk : 2 * tr.nchunk;  // at most 64 (checked on the host)
+  // headers, one partial per lane: (reference max, sum, visible count, true max)
+  const float4 h0 = lane < nparts ? ld_once(part(lane)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+  const float4 h1 = lane + 32 < nparts ? ld_once(part(lane + 32)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+  const float m = warp_max(fmaxf(h0.w, h1.w));  // true row max over the partials (base 2)
+  // weight of each partial; a partial that saw nothing (reference -inf) has
+  // weight 0 and an unwritten output
+  const float a0 = h0.x == -INFINITY ? 0.0f : exp2f(h0.x - m);
+  const float a1 = h1.x == -INFINITY ? 0.0f : exp2f(h1.x - m);
+  const float lsum = warp_sum(fmaf(h0.y, a0, h1.y * a1));
+  const float n = warp_sum(h0.z + h1.z);
   float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-  float lsum = 0.0f, n = 0.0f;
+  // outputs, four channels per lane, partials in order; the loads do not
+  // depend on each other
+#pragma unroll 8
   for (int k = 0; k < nparts; ++k) {
-    const float *p = part(k);
-    n += p[2];
-    if (p[0] == -INFINITY) continue;
-    float a = exp2f(p[0] - m);
-    lsum = fmaf(p[1], a, lsum);
-    float4 v = *reinterpret_cast<const float4 *>(p + 4 + lane * 4);
+    const float a = __shfl_sync(0xffffffffu, k < 32 ? a0 : a1, k & 31);
+    float4 v = ld_once(part(k) + 4 + lane * 4);
+    if (a == 0.0f) v = make_float4(0.f, 0.f, 0.f, 0.f);
     o.x = fmaf(v.x, a, o.x);
     o.y = fmaf(v.y, a, o.y);
     o.z = fmaf(v.z, a, o.z);
     o.w = fmaf(v.w, a, o.w);
   }
-  float inv = lsum > 0.0f ? 1.0f / lsum : 0.0f;
-  int h = kvh * L.g + row / tr.W, w = row % tr.W;
+  const float inv = lsum > 0.0f ? 1.0f / lsum : 0.0f;
+  const int h = kvh * L.g + row / tr.W, w = row % tr.W;
   float *dst = tr.stats + (((int64_t)l * L.Hq + h) * tr.W + w) * (D + 4);
-  if (lane == 0) *reinterpret_cast<float4 *>(dst) = make_float4(m == -INFINITY ? m : m * 0.69314718055994531f, lsum, n, 0.0f);
+  if (lane == 0)
+    *reinterpret_cast<float4 *>(dst) = make_float4(m == -INFINITY ? m : m * 0.69314718055994531f, lsum, n, 0.0f);
   *reinterpret_cast<float4 *>(dst + 4 + lane * 4) = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
+}
+
+// One warp per probe row of the selected layers (the two-launch path).
+__global__ void __launch_bounds__(256) combine_tc(const __grid_constant__ TcLaunch L) {
+  const int gw = (blockIdx.x * 256 + threadIdx.x) / 32, lane = threadIdx.x % 32;
+  if (gw >= L.row_off[L.n_traj]) return;
+  const int t = traj_of(L.row_off, L.n_traj, gw);
+  const TcTraj &tr = L.t[t];
+  int local = gw - L.row_off[t];
+  const int rows = L.g * tr.W;
+  const int row = local % rows;
+  local /= rows;
+  merge_row<false>(L, t, local / L.H, local % L.H, row, lane);
 }
 
 // ============================================================== prep
@@ -690,8 +896,9 @@ __device__ __forceinline__ ItemB decode_b(const TcLaunch &L, int item) {
   return b;
 }
 
-__global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
-  extern __shared__ uint8_t smem_raw[];
+template <bool FUSED>
+__device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint8_t *smem_raw, const int cta,
+                                          const int ncta) {
   SmemB &sm = *reinterpret_cast<SmemB *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_items = L.item_off_b[L.n_traj];
@@ -753,7 +960,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       uint32_t it = 0, n_local = 0, n_k = 0, n_v = 0;  // tiles; Q, K and V copies issued
       int po_base = 0;  // page ordinal of the item's first page
       bool stop = false;
-      for (int item = blockIdx.x; item < n_items && !stop; item += gridDim.x) {
+      for (int item = cta; item < n_items && !stop; item += ncta) {
         if (*abort_flag) break;
         ItemB bi = decode_b(L, item);
         if (bi.nslot == 0) continue;
@@ -868,7 +1075,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       if (lane == 0) {
         uint32_t it = 0;
         bool ok = true;
-        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        for (int item = cta; item < n_items && ok; item += ncta) {
           ItemB bi = decode_b(L, item);
           if (bi.nslot == 0) continue;
           int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
@@ -914,7 +1121,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       if (lane == 0) {
         uint32_t it = 0, n_local = 0;
         bool ok = true;
-        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        for (int item = cta; item < n_items && ok; item += ncta) {
           ItemB bi = decode_b(L, item);
           if (bi.nslot == 0) continue;
           int ntile = (bi.nslot + SLOTS - 1) / SLOTS;
@@ -954,7 +1161,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     float S_cur = 0.0f;
     int n_cur = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+    for (int item = cta; item < n_items && ok; item += ncta) {
       ItemB bi = decode_b(L, item);
       if (bi.nslot == 0) continue;
       const TcTraj &tr = L.t[bi.t];
@@ -962,6 +1169,11 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       int grow = bi.rt * BM + row;
       bool valid_row = grow < rows;
       int qp = -0x7fffffff;
+      // the row stats of this slice are complete once every share is merged
+      if (FUSED && !warp_poll_geq(&L.merged[slice_of(L, bi)], 4u * items_per_slice(L, bi.t), abort_flag, hdr)) {
+        ok = false;
+        break;
+      }
       // rows outside the slice, or rows that see nothing, get e = 0 everywhere
       float neg_m2 = -INFINITY;
       if (valid_row) {
@@ -1088,7 +1300,7 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
     const uint32_t u_col = 2 * BT + par * D;
     int po = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+    for (int item = cta; item < n_items && ok; item += ncta) {
       ItemB bi = decode_b(L, item);
       if (bi.nslot == 0) continue;
       const TcTraj &tr = L.t[bi.t];
@@ -1096,6 +1308,10 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
       int grow = bi.rt * BM + row;
       bool valid_row = grow < rows;
       int h = bi.kvh * L.g + (valid_row ? grow / tr.W : 0), w = valid_row ? grow % tr.W : 0;
+      if (FUSED && !warp_poll_geq(&L.merged[slice_of(L, bi)], 4u * items_per_slice(L, bi.t), abort_flag, hdr)) {
+        ok = false;
+        break;
+      }
       float2 o2[D / 2];
       float lsum = 0.0f, onorm = 0.0f;
       int nvis = 0;
@@ -1108,7 +1324,11 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
 #pragma unroll
         for (int c = 0; c < D; c += 4) {
           float4 v = valid_row ? *reinterpret_cast<const float4 *>(st + 4 + c) : make_float4(0.f, 0.f, 0.f, 0.f);
-          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+          // explicit FMAs: the same rounding in every kernel this body is compiled into
+          ss = fmaf(v.x, v.x, ss);
+          ss = fmaf(v.y, v.y, ss);
+          ss = fmaf(v.z, v.z, ss);
+          ss = fmaf(v.w, v.w, ss);
           o2[c / 2] = make_float2(v.x, v.y);
           o2[c / 2 + 1] = make_float2(v.z, v.w);
         }
@@ -1164,8 +1384,30 @@ __global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLa
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tm, 512);
-  if (threadIdx.x == 0 && sm.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, 11);
+  if (threadIdx.x == 0 && sm.abort_flag) {
+    if (FUSED) atomicExch(&hdr->abort, 1);
+    record_error(hdr, COMMITKV_ERR_TIMEOUT, 11);
+  }
 }
+
+__global__ void __launch_bounds__(512, 1) pass_b_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  page_body<false>(L, hdr, smem_raw, blockIdx.x, gridDim.x);
+}
+
+// ============================================================== fused
+// One cooperative launch over all SMs: CTAs [0, n_a) run the flash pass
+// (and merge the row stats slice by slice), CTAs [n_a, grid) run the page
+// pass, each page-pass item waiting until its slice's stats are merged.
+// Items of both passes are taken in slice order, so the page pass re-reads
+// a slice's keys and values shortly after the flash pass read them, while
+// they are still in L2.  Every cross-CTA wait is bounded.
+__global__ void __launch_bounds__(512, 1) score_fused_tc(const __grid_constant__ TcLaunch L, WsHeader *hdr) {
+  extern __shared__ uint8_t smem_raw[];
+  if ((int)blockIdx.x < L.n_a) flash_body<true>(L, hdr, smem_raw, blockIdx.x, L.n_a);
+  else page_body<true>(L, hdr, smem_raw, blockIdx.x - L.n_a, gridDim.x - L.n_a);
+}
+
 
 // ============================================================== host side
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -1221,18 +1463,71 @@ bool build_maps(TcMaps &mp, const TrajDev &t, int M, int H, int Hq) {
   return ok;
 }
 
-cudaError_t launch_score_tc(const TcLaunch &L, WsHeader *hdr, cudaStream_t s, int sm_count) {
-  cudaError_t e = cudaFuncSetAttribute(pass_a_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_a());
+int fused_chunk_len(int max_tokens, int max_row_tiles) {
+  // about kFusedItemsPerSlice flash items per slice (row tiles included), at
+  // least 512 tokens each, whole 128-token tiles
+  const int64_t per = ((int64_t)max_tokens * max_row_tiles + kFusedItemsPerSlice - 1) / kFusedItemsPerSlice;
+  const int64_t c = per < 512 ? 512 : per;
+  return (int)((c + BT - 1) / BT * BT);
+}
+
+int fused_flash_ctas(const TcLaunch &L, int sm_count) {
+  int na = (int)(sm_count * kFusedFlashShare + 0.5);
+  if (const char *e = getenv("COMMITKV_FUSED_FLASH_CTAS")) na = atoi(e);  // tuning experiments
+  const int items_a = L.item_off_a[L.n_traj], items_b = L.item_off_b[L.n_traj];
+  if (items_b == 0) na = sm_count;
+  na = na < 1 ? 1 : na > sm_count - 1 ? sm_count - 1 : na;
+  // A partial slot is reused n_a * kRing items later, after the slice of its
+  // earlier item is merged.  That slice's items must all come earlier than
+  // the reusing item (else the wait could depend on itself): n_a * kRing
+  // must cover the items of any slice.
+  int nis_max = 1;
+  for (int t = 0; t < L.n_traj; ++t) {
+    const int nis = L.t[t].nchunk * L.t[t].nrt;
+    nis_max = nis > nis_max ? nis : nis_max;
+  }
+  const int na_min = (nis_max + kRing - 1) / kRing;
+  na = na < na_min ? na_min : na;
+  return na < items_a ? na : items_a;
+}
+
+cudaError_t launch_score_tc(TcLaunch &L, WsHeader *hdr, cudaStream_t s, int sm_count) {
+  cudaError_t e;
+  for (int t = 0; t < L.n_traj; ++t)
+    if (L.t[t].nchunk > 32) return cudaErrorInvalidValue;  // the row merge takes at most 64 partials
+  const int na_items = L.from_stats ? 0 : L.item_off_a[L.n_traj];
+  const int nb_items = L.item_off_b[L.n_traj];
+  if (L.fused && na_items > 0) {
+    // fused: prep, then one cooperative launch of both passes
+    const size_t smem = smem_a() > smem_b() ? smem_a() : smem_b();
+    e = cudaFuncSetAttribute(score_fused_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, score_fused_tc, 512, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm != 1) return cudaErrorInvalidConfiguration;  // one CTA per SM: all 512 TMEM columns each
+    L.n_a = fused_flash_ctas(L, sm_count);
+    int nb = sm_count - L.n_a;
+    nb = nb < nb_items ? nb : nb_items;
+    if (nb < 1 && nb_items > 0) return cudaErrorInvalidConfiguration;
+    prep_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
+    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaMemsetAsync(L.a_done, 0, (size_t)L.slice_off[L.n_traj] * kCounterStride * 4, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(L.merged, 0, (size_t)L.slice_off[L.n_traj] * kCounterStride * 4, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(&hdr->abort, 0, sizeof(int32_t), s);
+    if (e != cudaSuccess) return e;
+    void *args[] = {(void *)&L, (void *)&hdr};
+    return cudaLaunchCooperativeKernel((const void *)score_fused_tc, dim3(L.n_a + nb), dim3(512), args, smem, s);
+  }
+  e = cudaFuncSetAttribute(pass_a_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_a());
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(pass_b_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_b());
   if (e != cudaSuccess) return e;
   prep_kernel<<<L.n_traj, 1024, 0, s>>>(L, hdr);
-  int na = L.from_stats ? 0 : L.item_off_a[L.n_traj];
-  if (na > 0) pass_a_tc<<<na < sm_count ? na : sm_count, 384, smem_a(), s>>>(L, hdr);
-  int rows = L.from_stats ? 0 : L.row_off[L.n_traj];
+  if (na_items > 0) pass_a_tc<<<na_items < sm_count ? na_items : sm_count, 384, smem_a(), s>>>(L, hdr);
+  const int rows = L.from_stats ? 0 : L.row_off[L.n_traj];
   if (rows > 0) combine_tc<<<(rows * 32 + 255) / 256, 256, 0, s>>>(L);
-  int nb = L.item_off_b[L.n_traj];
-  if (nb > 0) pass_b_tc<<<nb < sm_count ? nb : sm_count, 512, smem_b(), s>>>(L, hdr);
+  if (nb_items > 0) pass_b_tc<<<nb_items < sm_count ? nb_items : sm_count, 512, smem_b(), s>>>(L, hdr);
   return cudaGetLastError();
 }
 

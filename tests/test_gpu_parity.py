@@ -649,6 +649,31 @@ def test_scoring_paths_agree(name, seed, monkeypatch):
     _assert_close(a[:, 0], s_[:, 0], 1e-5, "row max")
 
 
+@pytest.mark.parametrize("name,seed", [("small", 0), ("small_w40_g16", 2), ("small_long_pages", 4)])
+def test_fused_and_two_launch_scoring_agree(name, seed, monkeypatch):
+    """The tensor-core scoring as one cooperative launch of both passes (the
+    default) and as separate flash, merge and page launches: effects within
+    the bf16 tolerance, visible counts and row maxima alike, and both
+    against the oracle."""
+    r = get_run(name, seed)
+    b, dev, o = r.buf, r.dev, r.orc
+    out = {}
+    for fused in ("1", "0"):
+        monkeypatch.setenv("COMMITKV_FUSED", fused)
+        R = torch.zeros(dev.P_post, device="cuda")
+        st = torch.zeros_like(b.stats[0])
+        ck.commitkv_page_effects(b.shape, [dev.post()], [R], stats_out=[st], workspace=b.ws)
+        torch.cuda.synchronize()
+        assert b.status() == ck.COMMITKV_OK
+        out[fused] = (_np(R), _np(st).reshape(-1, r.cfg.d + 4))
+        _assert_close(out[fused][0], o.R_post, r.tol, f"R+ (fused={fused}) against the oracle")
+    _assert_close(out["1"][0], out["0"][0], 2e-2, "R+ fused vs two launches")
+    a, c = out["1"][1], out["0"][1]
+    assert np.array_equal(a[:, 2], c[:, 2])
+    _assert_close(a[:, 0], c[:, 0], 1e-6, "row max")
+    _assert_close(a[:, 1], c[:, 1], 1e-5, "row sum")
+
+
 def test_many_zero_length_pages():
     """Zero-length pages take no slot: an item may hold more pages than its
     slots.  Their effect is 0; the other pages are unaffected."""
