@@ -15,6 +15,9 @@ commits, in the order of Algorithm 1, with plain Python bookkeeping:
                filled by the caller's per-token score, and K, V, positions are
                gathered.  A page keeps the tokens of it that are retained; its
                span is found again from the retained indices.
+  decode_checkpoint  the same on the decode cadence, the fill score being
+               each resident token's largest attention weight from the latest
+               window (reading 13b, core.token_scores).
   post_commit  R+ over the post-commit window; E_c = the pages measured at
                the pre-commit that are still resident and not retired;
                classification (Eq. 9-10), at most scan_cap candidates in
@@ -91,8 +94,23 @@ class OracleSession:
 
     # ---------------------------------------------------------------- checkpoint
     def checkpoint(self, fill_by_pos):
-        """Eq. 12-13 and Eq. 4 at a compression checkpoint: returns I (old
-        resident indices, ascending)."""
+        """Eq. 12-13 and Eq. 4 at a compression checkpoint, the budget filled
+        by a score per absolute position: returns I (old resident indices,
+        ascending)."""
+        return self.checkpoint_resident(np.asarray(fill_by_pos, np.float32)[self.pos])
+
+    def fill_scores(self, Q, qpos):
+        """The self-contained fill score of every resident token (reading
+        13b): its largest attention weight from the window (Q, qpos)."""
+        return core.token_scores(self._problem(Q, qpos))
+
+    def decode_checkpoint(self, Q, qpos):
+        """A checkpoint on the decode cadence (the paper compresses every 128
+        decoded tokens), the budget filled by the window's attention."""
+        return self.checkpoint_resident(self.fill_scores(Q, qpos))
+
+    def checkpoint_resident(self, fill):
+        """Eq. 12-13 and Eq. 4 with a fill score per resident token."""
         S = self.pos.shape[0]
         ids = self.page_ids()
         ps = np.asarray([p[1] for p in self.pages], np.int64)
@@ -100,7 +118,7 @@ class OracleSession:
         retired = np.asarray([pid in self.retired for pid in ids], np.uint8)
         pend = [i for i, pid in enumerate(ids) if pid in set(self.measured)]
         prio = np.asarray([self.R_pre[ids[i]] for i in pend], np.float32)
-        fill = np.asarray(fill_by_pos, np.float32)[self.pos]
+        fill = np.asarray(fill, np.float32)
         I = core.select_indices(S, ps, pl, retired, np.asarray(pend, np.int64), prio, fill, self.B, self.B_N,
                                 self.protect_cap)
         self.K, self.V, pos = core.gather(self.K, self.V, self.pos, I)

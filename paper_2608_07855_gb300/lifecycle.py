@@ -19,6 +19,11 @@ library's entry points in the order of Algorithm 1:
                session's own buffers; page spans are found again from the
                retained indices (a page keeps whichever of its tokens are
                retained, which stay contiguous).
+  decode checkpoints  the paper's setting compresses every 128 decoded
+               tokens: append() counts the decoded tokens, checkpoint_due()
+               says when, and decode_checkpoint() fills the budget by each
+               resident token's largest attention weight from the latest
+               window (commitkv_token_scores on the window's row stats).
   post_commit  R+ over the post-commit window with the row stats;
                classification (Eq. 9-10, or an ablation variant of Section
                4.4); at most scan_cap candidates in order (the paper scans at
@@ -49,7 +54,7 @@ def _torch():
 class Session:
     def __init__(self, shape: ck.Shape, G: int, B: int, eta: float, capacity: int, scan_cap: int = 64,
                  protect_cap: int = 16, thresholds: ck.Thresholds = None, variant: int = 0,
-                 tau_joint: float = 0.05, device="cuda"):
+                 tau_joint: float = 0.05, checkpoint_every: int = 128, device="cuda"):
         torch = _torch()
         self.shape, self.G, self.B = shape, G, B
         self.B_N = int(math.floor(eta * B))
@@ -67,6 +72,8 @@ class Session:
         self.R_pre = {}       # page id -> R- (fp32) of the latest commit
         self.measured = []    # page ids waiting for their post-commit measurement
         self.retired = set()  # D_c: accepted page ids still resident
+        self.checkpoint_every = checkpoint_every  # decoded tokens between checkpoints (0: caller-driven only)
+        self.decoded_since = 0  # decoded tokens appended since the last checkpoint
         self.ws = None
 
     # ---------------------------------------------------------------- helpers
@@ -104,6 +111,7 @@ class Session:
             "K": self.K[:, :, :S].clone(), "V": self.V[:, :, :S].clone(), "pos": self.pos[:S].clone(),
             "pages": [list(p) for p in self.pages], "next_id": self.next_id,
             "R_pre": dict(self.R_pre), "measured": list(self.measured), "retired": sorted(self.retired),
+            "decoded_since": self.decoded_since,
         }
 
     def load_state_dict(self, st):
@@ -124,19 +132,24 @@ class Session:
         self.R_pre = dict(st["R_pre"])
         self.measured = list(st["measured"])
         self.retired = set(st["retired"])
+        self.decoded_since = int(st.get("decoded_since", 0))
 
     def _config(self):
         s, th = self.shape, self.thresholds
         return {"shape": (s.layers, s.kv_heads, s.q_heads, s.head_dim, s.dtype, float(s.softmax_scale)),
                 "G": self.G, "B": self.B, "B_N": self.B_N, "scan_cap": self.scan_cap,
                 "protect_cap": self.protect_cap, "variant": int(self.variant), "tau_joint": float(self.tau_joint),
+                "checkpoint_every": int(self.checkpoint_every),
                 "thresholds": None if th is None else (th.tau_use, th.tau_dead, th.rho_use, th.rho_dead)}
 
     # ---------------------------------------------------------------- cache
-    def append(self, K, V, pos, events):
+    def append(self, K, V, pos, events, decoded: int = 0):
         """Append n resident tokens: K, V [M][H][n][d] and absolute
         positions [n] (device tensors); events = [(kind, first position,
-        length)] of the tool calls and observations inside them."""
+        length)] of the tool calls and observations inside them; decoded =
+        how many of the n the model decoded (reasoning, tool calls), for the
+        checkpoint cadence."""
+        self.decoded_since += int(decoded)
         n = int(pos.shape[0])
         if self.S + n > self.cap:
             raise ValueError("session capacity exceeded")
@@ -168,6 +181,37 @@ class Session:
         self.R_pre = dict(zip(ids, Rh))
         self.measured = [pid for pid in ids if pid not in self.retired]
         return R[:len(self.pages)]
+
+    def checkpoint_due(self) -> bool:
+        """Whether the decode cadence calls for a checkpoint now: at least
+        checkpoint_every decoded tokens since the last one (the paper's
+        setting compresses every 128 decoded tokens) and more resident
+        tokens than the budget."""
+        return self.checkpoint_every > 0 and self.decoded_since >= self.checkpoint_every and self.S > self.B
+
+    def fill_scores(self, Q, qpos):
+        """Self-contained fill scores (device float [S]): each resident
+        token's largest attention weight from the window Q [M][Hq][W][d],
+        qpos [W] (commitkv_page_effects on the cache without pages for the
+        window's row stats, then commitkv_token_scores)."""
+        torch = _torch()
+        s = self.shape
+        S = self.S
+        none = torch.zeros(0, dtype=torch.int32, device=self.dev)
+        tr = ck.TrajTensors(self.K[:, :, :S], self.V[:, :, :S], self.pos[:S], Q, qpos, none, none)
+        ws = self._workspace(self._traj())
+        stats = torch.zeros(s.layers, s.q_heads, Q.shape[2], s.head_dim + 4, device=self.dev)
+        R = torch.zeros(1, device=self.dev)
+        ck.commitkv_page_effects(s, [tr], [R], stats_out=[stats], workspace=ws)
+        scores = torch.zeros(max(S, 1), device=self.dev)
+        ck.commitkv_token_scores(s, [tr], [stats], [scores[:S]], workspace=ws)
+        self._check()
+        return scores[:S]
+
+    def decode_checkpoint(self, Q, qpos):
+        """A checkpoint on the decode cadence, the budget filled by the
+        window's attention (fill_scores).  Returns the retained indices."""
+        return self.checkpoint(self.fill_scores(Q, qpos))
 
     def checkpoint(self, fill):
         """Compression checkpoint (Eq. 12-13, Eq. 4): fill = device float
@@ -202,6 +246,7 @@ class Session:
                 pages.append([pid, kept[0], len(kept)])
         self.pages, self.S = pages, n
         self.retired &= set(self.page_ids())
+        self.decoded_since = 0
         return idx[:n]
 
     def post_commit(self, Q, qpos):

@@ -529,6 +529,7 @@ class Timeline:
     Q_pre: np.ndarray = None
     Q_post: np.ndarray = None
     fill: np.ndarray = None
+    Q_tok: np.ndarray = None  # [S][M][Hq][d]: the query each position decodes with (decode-cadence windows)
 
     @property
     def S(self):
@@ -540,6 +541,23 @@ class Timeline:
 
     def qpos_post(self, t):
         return np.arange(self.post_start[t], self.post_start[t] + self.cfg.W, dtype=np.int32)
+
+    def decoded(self, a, b):
+        """Decoded tokens in positions [a, b): the model writes the reasoning
+        and tool-call events; the query and the observations are prefilled."""
+        n = 0
+        for kind, s, m in self.events:
+            if kind in ("reason", "call"):
+                n += max(0, min(b, s + m) - max(a, s))
+        return n
+
+    def window(self, end):
+        """The probe window of a decode-cadence checkpoint taken when
+        position end - 1 has just been decoded: the queries of the last W
+        positions, as ([M][Hq][W][d], positions [W])."""
+        W = self.cfg.W
+        q = np.ascontiguousarray(np.transpose(self.Q_tok[end - W:end], (1, 2, 0, 3)))
+        return q, np.arange(end - W, end, dtype=np.int32)
 
 
 def make_timeline(cfg: Config, seed: int = 0, turns: int = 3, values: bool = True) -> Timeline:
@@ -573,23 +591,51 @@ def make_timeline(cfg: Config, seed: int = 0, turns: int = 3, values: bool = Tru
         tl.Q_pre = normal(seed, _stream(0, _T_TIMELINE + 3), (turns, M, Hq, W, d), bf16=bf)
         tl.Q_post = normal(seed, _stream(0, _T_TIMELINE + 4), (turns, M, Hq, W, d), bf16=bf)
         tl.fill = uniform_array(seed, _stream(0, _T_TIMELINE + 5), S)
+        tl.Q_tok = normal(seed, _stream(0, _T_TIMELINE + 6), (S, M, Hq, d), bf16=bf)
     return tl
 
 
-def timeline_steps(tl: Timeline):
+def timeline_steps(tl: Timeline, decode_every: int = 0):
     """The order in which a timeline is fed to a lifecycle session:
     ("append", a, b) the tokens [a, b); ("pre", t) commit t's pre-commit
     measurement; ("checkpoint",) a compression checkpoint (taken when the
     resident tokens exceed the budget); ("post", t) commit t's post-commit
-    measurement and decisions."""
+    measurement and decisions.  With decode_every > 0, appends are also cut
+    at the end of the first reasoning or tool-call event after every
+    decode_every decoded tokens (Timeline.decoded), and ("decode_checkpoint",
+    end) follows each such cut: the compression cadence of the paper's
+    setting (every 128 decoded tokens), taken at event boundaries so that a
+    cut never splits an event's pages, its fill scored by the window of the
+    last W positions before end."""
     steps, t0 = [], 0
+    count, due = 0, decode_every
+
+    def append(a, b):
+        nonlocal count, due
+        if not decode_every:
+            steps.append(("append", a, b))
+            return
+        p = a
+        ends = sorted(s + n for kind, s, n in tl.events if kind in ("reason", "call") and a < s + n <= b)
+        for e in ends:
+            if count + tl.decoded(p, e) >= due and e >= tl.cfg.W:
+                count += tl.decoded(p, e)
+                steps.append(("append", p, e))
+                steps.append(("decode_checkpoint", e))
+                while due <= count:
+                    due += decode_every
+                p = e
+        if p < b:
+            count += tl.decoded(p, b)
+            steps.append(("append", p, b))
+
     for k in range(tl.turns):
-        steps.append(("append", t0, int(tl.commit_end[k])))
+        append(t0, int(tl.commit_end[k]))
         t0 = int(tl.commit_end[k])
         steps.append(("pre", k))
         steps.append(("checkpoint",))
         end = int(tl.post_start[k]) + tl.cfg.W
-        steps.append(("append", t0, end))
+        append(t0, end)
         t0 = end
         steps.append(("post", k))
     return steps

@@ -737,3 +737,62 @@ def test_qwen_shape_plain_normal_inputs():
     _assert_close(st[:, 1], l, 1e-4, "row sum")
     err = np.linalg.norm(st[:, 4:] - o_vec, axis=1) / np.maximum(np.linalg.norm(o_vec, axis=1), 1e-30)
     assert err.max() <= 1e-4, err.max()
+
+
+def _token_scores_close(got, want, tol, what):
+    """Token scores against the oracle: relative tol, exact zeros (tokens no
+    probe query sees); scores below 1e-30 (fp32 exponent range) count as 0."""
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    assert np.array_equal(got == 0, want < 1e-30), what + ": zeros differ"
+    ok = (np.abs(got - want) <= tol * np.abs(want)) | (want < 1e-30)
+    assert ok.all(), f"{what}: {int((~ok).sum())} of {ok.size} outside {tol}"
+
+
+@pytest.mark.parametrize("name,seed", [("tiny", 0), ("small", 0), ("small_w40_g16", 2), ("small_long_pages", 4),
+                                       ("small_f32", 3)])
+@pytest.mark.parametrize("window", ["pre", "post"])
+def test_token_scores(name, seed, window):
+    """Per-token fill scores (window attention, Eq. 13's fill) from the
+    GPU's own row stats of the same cache and window, against the oracle's
+    softmax written out row by row: every token, within the effect
+    tolerance; tokens no probe query sees score exactly 0."""
+    r = get_run(name, seed)
+    cfg, b, dev, o = r.cfg, r.buf, r.dev, r.orc
+    t = dev.pre() if window == "pre" else dev.post()
+    S = dev.tr.L_pre if window == "pre" else dev.tr.S_post
+    stats = torch.zeros_like(b.stats[0])
+    R = torch.zeros(max(dev.P_post, 1), device="cuda")
+    P = dev.P_pre if window == "pre" else dev.P_post
+    ck.commitkv_page_effects(b.shape, [t], [R[:P]], stats_out=[stats], workspace=b.ws)
+    scores = torch.full((S,), -1.0, device="cuda")
+    ck.commitkv_token_scores(b.shape, [t], [stats], [scores], workspace=b.ws)
+    torch.cuda.synchronize()
+    assert b.status() == ck.COMMITKV_OK
+    want = core.token_scores(o.pre if window == "pre" else o.post)
+    _token_scores_close(_np(scores), want, r.tol, f"token scores ({window})")
+
+
+def test_token_scores_layer_mask_and_paths(monkeypatch):
+    """One selected layer, and the CUDA-core kernel forced for bf16: both
+    against the oracle and against each other."""
+    r = get_run("small_w40_g16", 2)
+    cfg, b, dev = r.cfg, r.buf, r.dev
+    mask = np.zeros(cfg.M, np.uint8)
+    mask[1] = 1
+    stats = torch.zeros_like(b.stats[0])
+    ck.commitkv_page_effects(b.shape, [dev.post()], b.R_post, stats_out=[stats], layer_mask=mask, workspace=b.ws)
+    out = {}
+    for path in ("tc", "simt"):
+        monkeypatch.setenv("COMMITKV_SCORING", path)
+        sc = torch.zeros(dev.tr.S_post, device="cuda")
+        ck.commitkv_token_scores(b.shape, [dev.post()], [stats], [sc], layer_mask=mask, workspace=b.ws)
+        torch.cuda.synchronize()
+        assert b.status() == ck.COMMITKV_OK
+        out[path] = _np(sc)
+    from oracle_bridge import problems
+    _, post = problems(dev.tr, layer_mask=mask)
+    want = core.token_scores(post)
+    for path in out:
+        _token_scores_close(out[path], want, 2e-2, f"token scores, layer 1 only ({path})")
+    _token_scores_close(out["tc"], out["simt"].astype(np.float64), 2e-2, "tc vs simt")

@@ -70,3 +70,27 @@ def test_resume_refuses_other_settings_and_small_capacity():
                     device="cpu")
     with pytest.raises(ValueError):
         small.load_state_dict(st)
+
+
+def test_checkpoint_cadence_counter():
+    """The decode cadence: append() counts decoded tokens, checkpoint_due()
+    asks for a checkpoint once checkpoint_every of them are in and the
+    cache is over budget, and the counter travels in state_dict (CPU: the
+    device is the CPU, no library call is made)."""
+    import torch
+    from paper_2608_07855_gb300 import commitkv as ck
+    from paper_2608_07855_gb300.lifecycle import Session
+    shape = ck.Shape(1, 1, 1, 64, ck.COMMITKV_F32, 0.0)
+    s = Session(shape, G=16, B=40, eta=0.125, capacity=200, checkpoint_every=32, device="cpu")
+    z = torch.zeros(1, 1, 30, 64)
+    s.append(z, z, torch.arange(30, dtype=torch.int32), [], decoded=30)
+    assert not s.checkpoint_due()  # 30 < 32 decoded
+    s.append(z, z, torch.arange(30, 60, dtype=torch.int32), [], decoded=2)
+    assert s.checkpoint_due()  # 32 decoded, 60 > 40 resident
+    st = s.state_dict()
+    t = Session(shape, G=16, B=40, eta=0.125, capacity=200, checkpoint_every=32, device="cpu")
+    t.load_state_dict(st)
+    assert t.decoded_since == 32 and t.checkpoint_due()
+    u = Session(shape, G=16, B=100, eta=0.125, capacity=200, checkpoint_every=32, device="cpu")
+    u.append(z, z, torch.arange(30, dtype=torch.int32), [], decoded=40)
+    assert not u.checkpoint_due()  # within budget

@@ -160,3 +160,54 @@ def test_hand_worked_timeline_scan_cap():
                 assert not o.retired
                 return
     raise AssertionError("no post-commit step")
+
+
+def test_decode_cadence_steps():
+    """timeline_steps with a decode cadence: the same appends (cut further),
+    commits and checkpoints in the same order; a decode checkpoint after
+    each cut at the end of a reasoning or tool-call event once another
+    decode_every decoded tokens are in."""
+    cfg = synth.small_config("timeline", event_len=(24, 80), G=16, M=1, H=1, Hq=4)
+    tl = synth.make_timeline(cfg, 3, 4, values=False)
+    plain = synth.timeline_steps(tl)
+    steps = synth.timeline_steps(tl, 40)
+    assert [x for x in steps if x[0] not in ("append", "decode_checkpoint")] == \
+        [x for x in plain if x[0] != "append"]
+    ends = {s + n for k, s, n in tl.events if k in ("reason", "call")}
+    pos, last = 0, 0
+    n_dc = 0
+    for x in steps:
+        if x[0] == "append":
+            assert x[1] == pos
+            pos = x[2]
+        elif x[0] == "decode_checkpoint":
+            assert x[1] == pos and x[1] in ends
+            assert tl.decoded(last, x[1]) >= 40 or last == 0
+            last = x[1]
+            n_dc += 1
+    assert n_dc >= 3
+    assert pos == [x for x in plain if x[0] == "append"][-1][2]
+
+
+def test_oracle_decode_checkpoint_keeps_the_most_attended_tokens():
+    """A decode checkpoint fills the budget by the window's attention: among
+    the tokens that are neither retired nor protected, every kept token
+    scores at least as high as every dropped one (ties by index)."""
+    from oracle import core
+    cfg = synth.small_config("timeline", event_len=(24, 80), G=16, M=1, H=1, Hq=4)
+    tl = synth.make_timeline(cfg, 4, 3)
+    K64, V64 = synth.values_f64(tl.K, cfg.dtype), synth.values_f64(tl.V, cfg.dtype)
+    o = OracleSession(cfg.M, cfg.H, cfg.Hq, cfg.d, cfg.G, 160, 0.125, protect_cap=0, thresholds=TH)
+    end = int(tl.commit_end[1])
+    o.append(K64[:, :, :end], V64[:, :, :end], np.arange(end), synth.timeline_events(tl, 0, end))
+    q, qp = tl.window(end)
+    fill = o.fill_scores(synth.values_f64(q, cfg.dtype), qp)
+    assert fill.shape == (end,) and (fill > 0).all() and (fill <= 1).all()
+    pb = o._problem(synth.values_f64(q, cfg.dtype), qp)
+    assert np.array_equal(fill, core.token_scores(pb))
+    I = o.decode_checkpoint(synth.values_f64(q, cfg.dtype), qp)
+    assert len(I) == 160
+    kept = np.zeros(end, bool)
+    kept[I] = True
+    f32 = fill.astype(np.float32)
+    assert f32[kept].min() >= f32[~kept].max()
