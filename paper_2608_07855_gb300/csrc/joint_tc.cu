@@ -258,7 +258,7 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const bool vis = rw.ok && i < nt[c] && s.pos[c][i] <= rw.qp;
-            const float e = vis ? exp2f(x[i] * b.scale_log2 - rw.m2) : 0.0f;
+            const float e = vis ? fast_exp2(fmaf(x[i], b.scale_log2, -rw.m2)) : 0.0f;
             se += e;
             ne += vis ? 1 : 0;
             x[i] = e;
