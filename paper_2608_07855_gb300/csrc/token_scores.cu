@@ -9,13 +9,15 @@
 // probe windows the paper builds on.
 //
 // Tensor-core path (bf16, head_dim 128, 16-byte aligned rows): a persistent
-// kernel, one CTA of 192 threads per SM, items (trajectory, layer, KV head,
+// kernel, one CTA of 320 threads per SM, items (trajectory, layer, KV head,
 // token chunk, 128-row tile of probe rows), the row tiles of one chunk
 // adjacent so that their K re-reads hit L2.  Per 128-token tile of K:
 //   warp 0  TMA: Q tile once per item, K tiles through a 4-stage ring
 //   warp 1  D[token][row] = K Q^T (tcgen05, fp32 in TMEM, two buffers)
-//   warps 2..5  one thread per token (TMEM lane): for every row p,
-//           exp2(s c - m_p log2 e) / l_p on the visible rows, max, and one
+//   warps 2..9  two groups of four taking alternate tiles, one thread per
+//           token (TMEM lane): for every row p, 2^(s c - m_p log2 e -
+//           log2 l_p) on the rows that see the token (all of them for the
+//           tokens at or before the smallest window position), max, and one
 //           atomic max into the token's score.
 // K rows are the MMA's M operand, so each thread reads its own token's row
 // of scores and the max over probe rows needs no cross-thread reduction.
@@ -98,15 +100,14 @@ struct Smem {
   alignas(1024) uint8_t q[kTileBytes];
   alignas(1024) uint8_t k[NST][kTileBytes];
   // per epilogue warp: its own copy of the item's row terms (no cross-warp barrier)
-  float m2[4][BR];     // row max in base-2 units
-  float inv_l[4][BR];  // 1 / row sum
-  int qp[4][BR];       // window position of the row; INT_MIN: the row sees nothing
+  float mlog[8][BR];  // row max + log2(row sum), base 2; +inf: the row sees nothing
+  int qp[8][BR];      // window position of the row
   uint64_t q_full, q_empty, k_full[NST], k_empty[NST], d_full[2], d_empty[2], drain;
   uint32_t tmem;
   int abort_flag;
 };
 
-__global__ void __launch_bounds__(192, 1) token_scores_tc(const __grid_constant__ TsLaunch L, WsHeader *hdr) {
+__global__ void __launch_bounds__(320, 1) token_scores_tc(const __grid_constant__ TsLaunch L, WsHeader *hdr) {
   extern __shared__ uint8_t smem_raw[];
   Smem &sm = *reinterpret_cast<Smem *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -207,11 +208,14 @@ __global__ void __launch_bounds__(192, 1) token_scores_tc(const __grid_constant_
       }
     }
   } else {
-    // ---------------------------------------------------------------- epilogue (warps 2..5)
+    // ---------------------------------------------------------------- epilogue (warps 2..9)
+    // Two groups of four warps take alternate tiles (group 0 the even
+    // tiles in TMEM buffer 0, group 1 the odd ones in buffer 1).
     const int ew = warp - 2;          // this warp's copy of the row terms
-    const int wq = warp & 3;          // TMEM lane quarter: warps 2, 3, 4, 5 -> 2, 3, 0, 1
+    const int hb = ew >> 2;           // this group's tiles: g & 1 == hb
+    const int wq = warp & 3;          // TMEM lane quarter: warps 2..5 -> 2, 3, 0, 1; 6..9 -> 2, 3, 0, 1
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
-    float *m2 = sm.m2[ew], *inv_l = sm.inv_l[ew];
+    float *mlog = sm.mlog[ew];
     int *qp = sm.qp[ew];
     uint32_t g = 0;
     bool ok = true;
@@ -219,32 +223,39 @@ __global__ void __launch_bounds__(192, 1) token_scores_tc(const __grid_constant_
       const Item a = decode(L, item);
       const TsTraj &tr = L.t[a.t];
       const int rows = L.g * tr.W;
+      // e = 2^(s c - m log2 e - log2 l) = exp(s - m) / l; every row that
+      // sees anything sees the tokens at or before the smallest window
+      // position, which then need no per-row test
       __syncwarp();
+      int qmin = 0x7fffffff;
       for (int r = lane; r < BR; r += 32) {
         const int row = a.rt * BR + r;
-        float mm = -INFINITY, il = 0.0f;
-        int q = -0x7fffffff - 1;
+        float ml = INFINITY;
+        int q = 0x7fffffff;
         if (row < rows) {
           const int h = a.kvh * L.g + row / tr.W, w = row % tr.W;
           const float4 st = *reinterpret_cast<const float4 *>(tr.stats + (((int64_t)a.l * L.Hq + h) * tr.W + w) *
                                                                            (D + 4));
           if (st.y > 0.0f && st.x != -INFINITY) {  // a row that sees nothing scores no token
-            mm = st.x * 1.4426950408889634f;
-            il = 1.0f / st.y;
+            ml = fmaf(st.x, 1.4426950408889634f, log2f(st.y));
             q = tr.qpos[w];
           }
         }
-        m2[r] = mm;
-        inv_l[r] = il;
+        mlog[r] = ml;
         qp[r] = q;
+        qmin = min(qmin, q);
       }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) qmin = min(qmin, __shfl_xor_sync(0xffffffffu, qmin, o));
       __syncwarp();
       const int t0 = a.c * kTilesPerItem * BT, t1 = min(tr.S, t0 + kTilesPerItem * BT);
       for (int tok0 = t0; tok0 < t1; tok0 += BT, ++g) {
         const int b = g & 1;
+        if (b != hb) continue;
         const int i = tok0 + wq * 32 + lane;  // this thread's token
         const bool valid = i < t1;
         const int pi = valid ? tr.pos[i] : 0x7fffffff;
+        const bool seen_by_all = pi <= qmin;
         if (!__all_sync(0xffffffffu, mbar_wait(&sm.d_full[b], (g >> 1) & 1, kWait, abort_flag))) {
           ok = false;
           break;
@@ -256,11 +267,15 @@ __global__ void __launch_bounds__(192, 1) token_scores_tc(const __grid_constant_
           float x[32];
           tmem_ld32f(tm + lane_base + b * BR + c0, x);
           tmem_wait_ld();
+          if (__all_sync(0xffffffffu, seen_by_all)) {
 #pragma unroll
-          for (int r = 0; r < 32; ++r) {
-            const bool vis = pi <= qp[c0 + r];
-            const float e = fast_exp2(fmaf(x[r], L.scale_log2, -m2[c0 + r])) * inv_l[c0 + r];
-            best = vis ? fmaxf(best, e) : best;
+            for (int r = 0; r < 32; ++r) best = fmaxf(best, fast_exp2(fmaf(x[r], L.scale_log2, -mlog[c0 + r])));
+          } else {
+#pragma unroll
+            for (int r = 0; r < 32; ++r) {
+              const float e = fast_exp2(fmaf(x[r], L.scale_log2, -mlog[c0 + r]));
+              best = pi <= qp[c0 + r] ? fmaxf(best, e) : best;
+            }
           }
         }
         tc_fence_before();
@@ -391,7 +406,7 @@ cudaError_t launch_tc(const Batch &b, const float *const *stats, float *const *s
       if (active && !tc::build_maps(L.maps[i], x, b.M, b.H, b.Hq)) return cudaErrorInvalidValue;
     }
     const int n = L.item_off[nb];
-    if (n > 0) token_scores_tc<<<n < sm_count ? n : sm_count, 192, smem_bytes(), s>>>(L, hdr);
+    if (n > 0) token_scores_tc<<<n < sm_count ? n : sm_count, 320, smem_bytes(), s>>>(L, hdr);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
