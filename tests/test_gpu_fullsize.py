@@ -15,6 +15,8 @@ any size, on sampled trajectories of a batch:
     page counts, bit-exact;
   * the joint test restricted to one or two layers (the layer mask),
     against the oracle's greedy scan of the same layers over the full cache;
+  * the per-token fill scores of one or two layers, every token of the
+    sampled trajectories;
   * selection (seeded retired set, pending pages, seeded priorities) and
     the gather, bit-exact; the gather is checked on the sampled slices.
 Tolerances are the bf16 ones of the other parity tests (2e-2 relative for
@@ -241,3 +243,32 @@ def test_compact_fullsize(full):
                 assert np.array_equal(_np(k_out[t][l, kvh, :n].view(torch.uint16)), tr.K[l, kvh, I]), t
                 assert np.array_equal(_np(v_out[t][l, kvh, :n].view(torch.uint16)), tr.V[l, kvh, I]), t
     del k_out, v_out
+
+
+def test_token_scores_selected_layers(full):
+    """Per-token fill scores (commitkv_token_scores, the self-contained fill)
+    over the full post-commit caches of the batch with one or two layers
+    selected, from the GPU's own row statistics of those layers: every token
+    of the sampled trajectories against the oracle's softmax written out row
+    by row over the same layers (relative tolerance; tokens no probe query
+    sees score exactly 0), and every score of the batch a softmax weight."""
+    trs, cfg, devs, shape, ws = full["trs"], full["cfg"], full["devs"], full["shape"], full["ws"]
+    layers = JOINT_LAYERS.get(cfg.name, (3, 30))
+    mask = np.zeros(cfg.M, np.uint8)
+    mask[list(layers)] = 1
+    f32 = dict(dtype=torch.float32, device="cuda")
+    stats = [torch.zeros(cfg.M, cfg.Hq, cfg.W, cfg.d + 4, **f32) for tr in trs]
+    R = [torch.zeros(tr.P_post, **f32) for tr in trs]
+    ck.commitkv_page_effects(shape, [d.post() for d in devs], R, stats_out=stats, layer_mask=mask, workspace=ws)
+    scores = [torch.full((tr.S_post,), -1.0, **f32) for tr in trs]
+    ck.commitkv_token_scores(shape, [d.post() for d in devs], stats, scores, layer_mask=mask, workspace=ws)
+    torch.cuda.synchronize()
+    assert ck.commitkv_workspace_status(ws) == ck.COMMITKV_OK
+    for t, sc in enumerate(scores):
+        assert float(sc.min()) >= 0.0 and float(sc.max()) <= 1.0, t
+    for t in full["sample"]:
+        want = core.token_scores(_slice_problem(trs[t], 0, 0, True, layers=layers))
+        got = _np(scores[t]).astype(np.float64)
+        assert np.array_equal(got == 0, want < 1e-30), f"trajectory {t}: zeros differ"
+        ok = (np.abs(got - want) <= TOL * np.abs(want)) | (want < 1e-30)
+        assert ok.all(), f"trajectory {t}: {int((~ok).sum())} of {ok.size} token scores outside {TOL}"
