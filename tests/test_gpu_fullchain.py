@@ -1,7 +1,9 @@
-"""Whole-chain parity of one step of the Qwen3-8B-shaped 32K + 4K workload
-(36 layers, 32 query / 8 KV heads, head_dim 128, bf16), in the launch
-configuration the benchmark times (StepBuffers.step: one scoring call over
-both caches, classify, joint test, compaction), against the oracle:
+"""Whole-chain parity of one step of the Qwen3-8B-shaped workloads (36
+layers, 32 query / 8 KV heads, head_dim 128, bf16): 32K + 4K, 16K + 2K, and
+one trajectory of the 16 of the ragged batch, which runs with the other 15
+in the same launches.  The launch configuration is the one the benchmark
+times (StepBuffers.step: one scoring call over both caches of the batch,
+classify, joint test, compaction); against the oracle:
 
   * R- and R+ of every page over all 288 (layer, KV head) slices of each
     cache (Eq. 6-8), within the bf16 tolerance (2e-2 relative);
@@ -47,26 +49,32 @@ def _check(got, want, what):
                              + ", ".join(f"[{i}] gpu {got[i]:.6g} oracle {want[i]:.6g}" for i in bad))
 
 
-def test_full_chain_qwen3_8b_32k():
+# (workload, trajectory checked, least number of candidates the planted pages give)
+CHAINS = [("qwen3_8b_32k", 0, 100), ("qwen3_8b_16k", 0, 40), ("ragged16", 0, 20)]
+
+
+@pytest.mark.parametrize("name,t,min_cand", CHAINS)
+def test_full_chain(name, t, min_cand):
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     ck.load_library()
-    cfg = synth.CONFIGS["qwen3_8b_32k"]
-    tr = synth.make_trajectory(cfg, 0)
-    dev = DeviceTrajectory.upload(tr)
-    b = StepBuffers(cfg, [dev])
+    cfg = synth.CONFIGS[name]
+    trs = [synth.make_trajectory(cfg, 0, traj=i) for i in range(cfg.n_traj)]
+    devs = [DeviceTrajectory.upload(x) for x in trs]
+    b = StepBuffers(cfg, devs)
     b.step()
     torch.cuda.synchronize()
     assert b.status() == ck.COMMITKV_OK
-    Rm_g = _np(b.R_pre[0]).astype(np.float64)  # [P_post]; the observation's pages stay 0
-    Rp_g = _np(b.R_post[0]).astype(np.float64)
-    state_g = _np(b.state[0])
-    nc = int(b.n_cand[0])
-    cand_g = _np(b.cand[0])[:nc].astype(np.int64)
-    acc_g = _np(b.accepted[0])[:tr.P_post]
-    step_g = _np(b.step_R[0])[:nc]
-    n_idx = int(b.n_idx[0])
-    idx_g = _np(b.idx[0])[:n_idx]
-    k_out, v_out, pos_out = b.k_out[0], b.v_out[0], _np(b.pos_out[0])[:n_idx]
+    tr = trs[t]
+    Rm_g = _np(b.R_pre[t]).astype(np.float64)  # [P_post]; the observation's pages stay 0
+    Rp_g = _np(b.R_post[t]).astype(np.float64)
+    state_g = _np(b.state[t])
+    nc = int(b.n_cand[t])
+    cand_g = _np(b.cand[t])[:nc].astype(np.int64)
+    acc_g = _np(b.accepted[t])[:tr.P_post]
+    step_g = _np(b.step_R[t])[:nc]
+    n_idx = int(b.n_idx[t])
+    idx_g = _np(b.idx[t])[:n_idx]
+    k_out, v_out, pos_out = b.k_out[t], b.v_out[t], _np(b.pos_out[t])[:n_idx]
 
     # 1. effects of every page over every slice, one layer at a time
     f64 = lambda a: synth.values_f64(a, cfg.dtype)  # noqa: E731
@@ -98,7 +106,7 @@ def test_full_chain_qwen3_8b_32k():
     assert safe.any()
     assert np.array_equal(state_g[idx][safe], s_o[idx][safe])
     # the workload plants completion candidates: a realistic count of them
-    assert nc >= 100, nc
+    assert nc >= min_cand, nc
 
     # 3. joint test over all 36 layers on the GPU's candidate list
     del K, V, pre, post
