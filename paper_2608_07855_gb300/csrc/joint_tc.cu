@@ -162,13 +162,13 @@ __host__ __device__ constexpr int top_bit(int T) { return T >= 8 ? 3 : T >= 4 ? 
 
 // One pass over the pages list[0..n) (n <= kRound).  kScan: accumulates the
 // squared norms of the subset sums over the team's channels into ss, and
-// o's into on2; otherwise adds the pages' D_E into D_A in the workspace.
+// o's into on2 (even and odd channels apart); otherwise adds the pages' D_E into D_A in the workspace.
 // S_E and n_E of every page are left in Sc and nc.  Returns false on a
 // timeout.
 template <bool kScan>
 __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeader *hdr, const Group &G,
                                          const Row &rw, const int *list, int n, bool stage_q, uint32_t tm,
-                                         uint32_t lane_base, uint32_t &phase, float (&ss)[kCombos], float &on2,
+                                         uint32_t lane_base, uint32_t &phase, float2 (&ss)[kCombos], float2 &on2,
                                          float (&Sc)[kRound], int (&nc)[kRound]) {
   const Batch &b = L.batch;
   const TrajDev &tr = b.t[G.t];
@@ -253,14 +253,22 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
           const uint32_t addr = tm + lane_base + kColS + kCT * c;
           tmem_ld32f(addr, x);
           tmem_wait_ld();
-          float se = 0.0f;
+          // the chunk's visible tokens: positions increase along the page,
+          // so they are a prefix, whole unless the row's position cuts it
           int ne = 0;
+          if (rw.ok && nt[c] > 0) {
+            if (s.pos[c][nt[c] - 1] <= rw.qp) {
+              ne = nt[c];
+            } else {
+#pragma unroll 1
+              for (int i = 0; i < nt[c]; ++i) ne += s.pos[c][i] <= rw.qp ? 1 : 0;
+            }
+          }
+          float se = 0.0f;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const bool vis = rw.ok && i < nt[c] && s.pos[c][i] <= rw.qp;
-            const float e = vis ? fast_exp2(fmaf(x[i], b.scale_log2, -rw.m2)) : 0.0f;
+            const float e = i < ne ? fast_exp2(fmaf(x[i], b.scale_log2, -rw.m2)) : 0.0f;
             se += e;
-            ne += vis ? 1 : 0;
             x[i] = e;
           }
           if (h == 0) {
@@ -322,27 +330,35 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
           for (int c = 0; c < kRound; ++c)
             if (c < n) tmem_ld8(tm + lane_base + 64 * c + kSub * q, u[c]);
           tmem_wait_ld();
+          // two channels per packed instruction (an addition as a product
+          // with 1: the same rounding)
+          const float2 one2 = make_float2(1.0f, 1.0f);
 #pragma unroll
-          for (int i = 0; i < kSub; ++i) {
-            float de[kRound];
+          for (int i = 0; i < kSub; i += 2) {
+            const float2 o2 = make_float2(o[i], o[i + 1]);
+            float2 de[kRound];
 #pragma unroll
-            for (int c = 0; c < kRound; ++c) de[c] = c < n ? fmaf(-Sc[c], o[i], __uint_as_float(u[c][i])) : 0.0f;
+            for (int c = 0; c < kRound; ++c)
+              de[c] = c < n ? ffma2(make_float2(-Sc[c], -Sc[c]), o2,
+                                    make_float2(__uint_as_float(u[c][i]), __uint_as_float(u[c][i + 1])))
+                            : make_float2(0.0f, 0.0f);
             if constexpr (kScan) {
-              on2 = fmaf(o[i], o[i], on2);
-              float p[1 << kRound];
-              p[0] = da[i];
+              on2 = ffma2(o2, o2, on2);
+              float2 p[1 << kRound];
+              p[0] = make_float2(da[i], da[i + 1]);
 #pragma unroll
               for (int T = 1; T < (1 << kRound); ++T) {
                 if (T >= (1 << n)) break;  // subsets of the pass's pages only
-                p[T] = p[T & ~(1 << top_bit(T))] + de[top_bit(T)];
-                ss[T - 1] = fmaf(p[T], p[T], ss[T - 1]);
+                p[T] = ffma2(de[top_bit(T)], one2, p[T & ~(1 << top_bit(T))]);
+                ss[T - 1] = ffma2(p[T], p[T], ss[T - 1]);
               }
             } else {
-              float x = da[i];
+              float2 x = make_float2(da[i], da[i + 1]);
 #pragma unroll
               for (int c = 0; c < kRound; ++c)
-                if (c < n) x += de[c];
-              da[i] = x;
+                if (c < n) x = ffma2(de[c], one2, x);
+              da[i] = x.x;
+              da[i + 1] = x.y;
             }
           }
           if constexpr (!kScan) {
@@ -432,12 +448,13 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
       rw.nA = rw.ok ? (int)L.SA[rw.grow * 2 + 1] : 0;
       if (tid < 16) s.rmax[tid] = 0u;
 
-      float ss[kCombos], on2 = 0.0f, Sc[kRound];
+      float2 ss2[kCombos], on2p = make_float2(0.0f, 0.0f);
+      float Sc[kRound];
       int nc[kRound];
 #pragma unroll
-      for (int i = 0; i < kCombos; ++i) ss[i] = 0.0f;
+      for (int i = 0; i < kCombos; ++i) ss2[i] = make_float2(0.0f, 0.0f);
       if (nf > 0) {
-        if (!run_pass<false>(s, L, hdr, G, rw, fold, nf, true, tm, lane_base, phase, ss, on2, Sc, nc)) {
+        if (!run_pass<false>(s, L, hdr, G, rw, fold, nf, true, tm, lane_base, phase, ss2, on2p, Sc, nc)) {
           ok = false;
           break;
         }
@@ -452,11 +469,14 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
           L.SA[rw.grow * 2 + 1] = (float)rw.nA;
         }
       }
-      if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, ss, on2, Sc, nc)) {
+      if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, ss2, on2p, Sc, nc)) {
         ok = false;
         break;
       }
-      // team 1's channel sums to team 0
+      // the channel sums of the thread, then team 1's to team 0
+      float ss[kCombos], on2 = on2p.x + on2p.y;
+#pragma unroll
+      for (int i = 0; i < kCombos; ++i) ss[i] = ss2[i].x + ss2[i].y;
       if (tid >= kTeam) {
 #pragma unroll
         for (int i = 0; i < kCombos; ++i) s.part[i][tid - kTeam] = ss[i];
