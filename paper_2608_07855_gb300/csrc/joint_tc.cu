@@ -69,7 +69,9 @@ struct SmemJ {
   float part[kCombos + 1][kRows];  // team 1's sums of squares (and ||o||^2) for team 0
   int pos[kRound][kCT];
   unsigned rmax[16];
-  uint64_t bar;
+  uint64_t bar;       // Q K^T done (one issuing thread)
+  uint64_t bar_pv;    // P V done (two issuing threads)
+  uint64_t drain[2];  // an issuing thread's MMAs done (after an abort)
   uint32_t tmem;
   int abort_flag;
 };
@@ -127,9 +129,9 @@ __device__ __forceinline__ Group decode_group(const JointLaunch &L, int grp) {
   return G;
 }
 
-// Waits for the MMAs committed to the pass barrier; uniform over the block.
-__device__ __forceinline__ bool wait_mma(SmemJ &s, uint32_t &phase) {
-  bool ok = mbar_wait(&s.bar, phase, kWait, &s.abort_flag);
+// Waits for the MMAs committed to a pass barrier; uniform over the block.
+__device__ __forceinline__ bool wait_mma(SmemJ &s, uint64_t *bar, uint32_t &phase) {
+  bool ok = mbar_wait(bar, phase, kWait, &s.abort_flag);
   phase ^= 1u;
   ok = __syncthreads_and(ok) != 0;
   if (ok) tc_fence_after();
@@ -168,7 +170,8 @@ __host__ __device__ constexpr int top_bit(int T) { return T >= 8 ? 3 : T >= 4 ? 
 template <bool kScan>
 __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeader *hdr, const Group &G,
                                          const Row &rw, const int *list, int n, bool stage_q, uint32_t tm,
-                                         uint32_t lane_base, uint32_t &phase, float2 (&ss)[kCombos], float2 &on2,
+                                         uint32_t lane_base, uint32_t &phase, uint32_t &phase_pv,
+                                         float2 (&ss)[kCombos], float2 &on2,
                                          float (&Sc)[kRound], int (&nc)[kRound]) {
   const Batch &b = L.batch;
   const TrajDev &tr = b.t[G.t];
@@ -243,7 +246,7 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
             mma_bf16(tm + kColS, desc_kmajor(s.q, kQHalf, ks), desc_kmajor(s.k, kKHalf, ks), idesc, ks > 0);
           mma_commit(&s.bar);
         }
-        if (!wait_mma(s, phase)) return false;
+        if (!wait_mma(s, &s.bar, phase)) return false;
         // ---- e = exp(s - m) on the visible tokens; P over S (team t takes
         // the pages c = t mod 2)
 #pragma unroll 1
@@ -284,12 +287,13 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
         tc_fence_before();
         __syncthreads();
       }
-      // ---- U_E (+)= P V_E for channel half h
-      if (tid == 0) {
+      // ---- U_E (+)= P V_E for channel half h; two threads issue, the even
+      // and the odd pages (accumulators of their own), and both commit
+      if (tid == 0 || tid == 32) {
         tc_fence_after();
         const uint32_t idesc = idesc_bf16_f32(kRows, 64, 0, 1);
 #pragma unroll 1
-        for (int c = 0; c < n; ++c) {
+        for (int c = tid / 32; c < n; c += 2) {
           const int nks = max(1, (nt[c] + 15) / 16);
 #pragma unroll 1
           for (int ks = 0; ks < nks; ++ks) {
@@ -298,11 +302,11 @@ __device__ __forceinline__ bool run_pass(SmemJ &s, const JointLaunch &L, WsHeade
             mma_bf16_ts(tm + 64 * c, tm + p_col(c, ks, 1), bd, idesc, 1u);
           }
         }
-        mma_commit(&s.bar);
+        mma_commit(&s.bar_pv);
       }
       const bool last = j == nch - 1;
       if (last) stage_half(s, rw, L.DA, h);  // in flight while the MMAs run
-      if (!wait_mma(s, phase)) return false;
+      if (!wait_mma(s, &s.bar_pv, phase_pv)) return false;
       if (last) {
         cp_async_wait_all();  // the thread's own parts of the half buffers
         if (h == 0) {
@@ -397,6 +401,9 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
   if (tid == 0) {
     s.abort_flag = 0;
     mbar_init(&s.bar, 1);
+    mbar_init(&s.bar_pv, 2);
+    mbar_init(&s.drain[0], 1);
+    mbar_init(&s.drain[1], 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -409,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
   const uint32_t tm = s.tmem;
   // warps w and w + 4 (the two teams) reach TMEM lanes 32 (w mod 4) ..
   const uint32_t lane_base = (uint32_t)((warp % 4) * 32) << 16;
-  uint32_t phase = 0;
+  uint32_t phase = 0, phase_pv = 0;
   bool ok = true;
 
   const int rounds = joint::round_total(L);
@@ -454,7 +461,8 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
 #pragma unroll
       for (int i = 0; i < kCombos; ++i) ss2[i] = make_float2(0.0f, 0.0f);
       if (nf > 0) {
-        if (!run_pass<false>(s, L, hdr, G, rw, fold, nf, true, tm, lane_base, phase, ss2, on2p, Sc, nc)) {
+        if (!run_pass<false>(s, L, hdr, G, rw, fold, nf, true, tm, lane_base, phase, phase_pv, ss2, on2p, Sc,
+                             nc)) {
           ok = false;
           break;
         }
@@ -469,7 +477,8 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
           L.SA[rw.grow * 2 + 1] = (float)rw.nA;
         }
       }
-      if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, ss2, on2p, Sc, nc)) {
+      if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, phase_pv, ss2, on2p,
+                          Sc, nc)) {
         ok = false;
         break;
       }
@@ -523,7 +532,10 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
     if (tid == 0) {
       if (s.abort_flag) record_error(hdr, COMMITKV_ERR_TIMEOUT, -5);
       atomicExch(&hdr->abort, 1);
-      mbar_wait_drain(&s.bar, phase ^ 1u, kWait);
+    }
+    if (tid == 0 || tid == 32) {  // the issuing threads: every MMA of theirs has completed
+      mma_commit(&s.drain[tid / 32]);
+      mbar_wait_drain(&s.drain[tid / 32], 0, kWait);
     }
   }
   tc_fence_before();
