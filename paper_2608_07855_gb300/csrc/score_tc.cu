@@ -83,7 +83,7 @@ __device__ __forceinline__ uint64_t desc_v(const uint8_t *tile, int ks) {
 template <bool FUSED>
 __device__ __forceinline__ float *part_ptr(const TcLaunch &L, int item, int h, int row) {
   const int64_t slot = FUSED ? (int64_t)(item % (L.n_a * kRing)) : (int64_t)item;
-  return L.partials + ((slot * 2 + h) * BM + row) * (D + 4);
+  return L.partials + ((slot * kPartsPerItem + h) * BM + row) * (D + 4);
 }
 
 // Index of an item's (trajectory, layer, KV head) slice in the per-slice counters.
@@ -531,7 +531,7 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
         if (lane == 0) mbar_arrive(&sm.p_full[b]);
       }
       if (!ok) break;
-      if (FUSED) {
+      {
         // One partial per item: warpgroup 1 publishes its (reference max,
         // sum, count, true max) and leaves its O in tensor memory; warpgroup
         // 0 rescales both outputs to the larger reference max, writes the
@@ -552,7 +552,7 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.pub_full);
         } else {
-          if (item >= L.n_a * kRing) {
+          if (FUSED && item >= L.n_a * kRing) {
             // the partial slot was last used by this CTA's item kRing items
             // back: its slice must be merged before the slot is overwritten
             const ItemA pa = decode_a(L, item - L.n_a * kRing);
@@ -584,11 +584,15 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
             tmem_wait_ld();
             if (valid_row) {
 #pragma unroll
-              for (int i = 0; i < 32; i += 4)
-                st_keep(dst + 4 + c0 + i, make_float4(fmaf(x0[i], f0, theirs ? x1[i] * f1 : 0.0f),
-                                                      fmaf(x0[i + 1], f0, theirs ? x1[i + 1] * f1 : 0.0f),
-                                                      fmaf(x0[i + 2], f0, theirs ? x1[i + 2] * f1 : 0.0f),
-                                                      fmaf(x0[i + 3], f0, theirs ? x1[i + 3] * f1 : 0.0f)));
+              for (int i = 0; i < 32; i += 4) {
+                const float4 v = make_float4(fmaf(x0[i], f0, theirs ? x1[i] * f1 : 0.0f),
+                                             fmaf(x0[i + 1], f0, theirs ? x1[i + 1] * f1 : 0.0f),
+                                             fmaf(x0[i + 2], f0, theirs ? x1[i + 2] * f1 : 0.0f),
+                                             fmaf(x0[i + 3], f0, theirs ? x1[i + 3] * f1 : 0.0f));
+                // the fused launch's merge reads the partial soon: keep it in L2
+                if (FUSED) st_keep(dst + 4 + c0 + i, v);
+                else *reinterpret_cast<float4 *>(dst + 4 + c0 + i) = v;
+              }
             }
           }
           tc_fence_before();
@@ -600,43 +604,16 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
           }
           if (mine) ++uses;
           // (reference max of l and O, sum, visible count, true max)
-          if (valid_row)
-            st_keep(dst, make_float4(mr, fmaf(lsum, f0, o1.y * f1), (float)nvis + o1.z, fmaxf(m_true, o1.w)));
-          signal_add(&L.a_done[slice_of(L, a)], lane);  // this warp's rows of the partial are written
+          if (valid_row) {
+            const float4 hd = make_float4(mr, fmaf(lsum, f0, o1.y * f1), (float)nvis + o1.z, fmaxf(m_true, o1.w));
+            if (FUSED) st_keep(dst, hd);
+            else *reinterpret_cast<float4 *>(dst) = hd;
+          }
+          if (FUSED) signal_add(&L.a_done[slice_of(L, a)], lane);  // this warp's rows of the partial are written
         }
         ++n_it;
         it += ntile;
-        continue;
       }
-      if (j0 < ntile) {
-        // this warpgroup's O is complete after its last P V of the item
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm.o_full[hb], uses & 1, kWait, abort_flag))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-#pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32(tm + lane_base + o_col + c0, r);
-          tmem_wait_ld();
-          if (valid_row) {
-#pragma unroll
-            for (int i = 0; i < 32; i += 4)
-              *reinterpret_cast<float4 *>(dst + 4 + c0 + i) =
-                  make_float4(__uint_as_float(r[i]), __uint_as_float(r[i + 1]), __uint_as_float(r[i + 2]),
-                              __uint_as_float(r[i + 3]));
-          }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.o_empty[hb]);
-        ++uses;
-      }
-      // (reference max of l and O, sum, visible count, true max); a warpgroup
-      // without tiles in this item leaves an empty partial
-      if (valid_row) *reinterpret_cast<float4 *>(dst) = make_float4(m_used, lsum, (float)nvis, m_true);
-      it += ntile;
     }
   } else if (FUSED) {
     // ------------------------------------------------------------ merge (warps 12..15, fused launch only)
@@ -681,14 +658,13 @@ __device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int 
   const TcTraj &tr = L.t[t];
   const int l = L.layer_ids[li];
   const int rt = row / BM, rl = row % BM;
-  // fused launch: partial k = chunk k (one per item); otherwise partial
-  // k = 2 c + h: chunk c, softmax warpgroup h
+  // partial k = chunk k (one per item: the two softmax warpgroups' states
+  // are merged in the CTA)
   auto part = [&](int k) {
-    const int c = FUSED ? k : k >> 1;
-    const int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + c) * tr.nrt + rt;
-    return part_ptr<FUSED>(L, item, FUSED ? 0 : k & 1, rl);
+    const int item = L.item_off_a[t] + ((li * L.H + kvh) * tr.nchunk + k) * tr.nrt + rt;
+    return part_ptr<FUSED>(L, item, 0, rl);
   };
-  const int nparts = FUSED ? tr.nchunk : 2 * tr.nchunk;  // at most 64 (checked on the host)
+  const int nparts = tr.nchunk;  // at most 32 (checked on the host)
   // headers, one partial per lane: (reference max, sum, visible count, true max)
   const float4 h0 = lane < nparts ? ld_once(part(lane)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
   const float4 h1 = lane + 32 < nparts ? ld_once(part(lane + 32)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);

@@ -11,7 +11,7 @@ namespace tc {
 constexpr int kMaxTc = 16;          // trajectories per launch (tensor maps travel as parameters)
 constexpr int kRowsPerTile = 128;   // probe rows per MMA tile
 constexpr int kSlotsPerItem = 128;  // 16-token slots per pass-B work item
-constexpr int kPartsPerItem = 2;    // pass-A partials per work item
+constexpr int kPartsPerItem = 1;    // pass-A partials per work item (the two softmax groups merged)
 constexpr int kPartialRing = 4;     // partial slots (items) per flash CTA of the fused launch
 constexpr int kMaxFusedCtas = 256;  // bound on the fused launch's flash CTAs (workspace sizing)
 constexpr int kFusedItemsPerSlice = 32;    // flash items per slice in the fused launch (chunking target)
