@@ -257,10 +257,11 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
 
   // warpgroup 0: TMA producer, P V issuer, Q K^T issuer, one idle warp; 1 and
   // 2: softmax of the even and the odd tiles.  Register budget per thread:
-  // 56 + 2 x 224 = the launch's 3 x 168.
+  // 104 + 2 x 200 = the launch's 3 x 168 (the issuers' loops spill below 104;
+  // the softmax needs no more than 200).
   if (warp < 4) {
     if (FUSED) regs_dec<48>();
-    else regs_dec<56>();  // warp 3 stays idle
+    else regs_dec<104>();  // warp 3 stays idle
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
       if (lane == 0) {
@@ -397,7 +398,7 @@ __device__ __forceinline__ void flash_body(const TcLaunch &L, WsHeader *hdr, uin
   } else if (warp < 12) {
     // ------------------------------------------------------------ softmax (warps 4..11)
     if (FUSED) regs_inc<208>();
-    else regs_inc<224>();
+    else regs_inc<200>();
     const int hb = (warp - 4) >> 2;   // this warpgroup's tiles: g & 1 == hb
     const int wq = warp & 3;          // TMEM lane quarter of this warp
     const int row = wq * 32 + lane;   // probe row within the tile
@@ -841,7 +842,7 @@ struct SmemB {
   int fifo_n[NFIFO][BM];    // per page: visible count of every row
   int fifo_page[NFIFO];
   uint64_t q_full, q_empty, k_full[NKB], k_empty[NKB], meta_empty[NKB], v_full[NVB], v_empty[NVB], s_full[2],
-      s_empty[2], p_full[2], acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain, drain2;
+      s_empty[2], p_full[2], acc_full[2], acc_empty[2], fifo_full[NFIFO], fifo_empty[NFIFO], drain[2], drain2;
   uint32_t tmem;
   int abort_flag;
 };
@@ -887,15 +888,15 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
     for (int s = 0; s < NKB; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.k_empty[s], 1);
-      mbar_init(&sm.meta_empty[s], 5);  // four softmax warps and the MMA thread
+      mbar_init(&sm.meta_empty[s], 6);  // four softmax warps and the two P V threads
     }
     for (int s = 0; s < NVB; ++s) {
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.v_empty[s], 1);
+      mbar_init(&sm.v_empty[s], 2);  // both P V threads
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&sm.s_full[b], 1);
-      mbar_init(&sm.s_empty[b], 1);
+      mbar_init(&sm.s_empty[b], 2);  // both P V threads
       mbar_init(&sm.acc_full[b], 1);
       mbar_init(&sm.acc_empty[b], 4);  // the epilogue warpgroup of that page parity
     }
@@ -908,7 +909,8 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
       mbar_init(&sm.fifo_full[f], 4);
       mbar_init(&sm.fifo_empty[f], 4);
     }
-    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain[0], 1);
+    mbar_init(&sm.drain[1], 1);
     mbar_init(&sm.drain2, 1);
     fence_mbar_init();
   }
@@ -921,12 +923,12 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
   tc_fence_after();
   const uint32_t tm = sm.tmem;
 
-  // warpgroup 0: TMA producer, P V issuer, Q K^T issuer, one idle warp; 1: softmax;
+  // warpgroup 0: TMA producer, two P V issuers (warps 1 and 3), Q K^T issuer; 1: softmax;
   // 2 and 3: epilogue.  Each branch first sets its warpgroup's register
   // budget: 64 + 112 + 2 x 168 per thread = the launch's 4 x 128 (a budget
   // below 128 is set with a decrease, above it with an increase).
   if (warp < 4) {
-    regs_dec<64>();  // warp 3 stays idle
+    regs_dec<64>();
     if (warp == 0) {
       // ------------------------------------------------------------ TMA producer
       // The whole warp works each tile: lanes 0..7 take one 16-token slot each
@@ -1046,8 +1048,12 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
           mbar_wait_drain(&sm.v_full[u % NVB], (u / NVB) & 1, kWait);
         if (n_local > 0) mbar_wait_drain(&sm.q_full, (n_local - 1) & 1, kWait);
       }
-    } else if (warp == 1) {
-      // ------------------------------------------------------------ P V issuer
+    } else if (warp == 1 || warp == 3) {
+      // ------------------------------------------------------------ P V issuers
+      // Two issuing threads, one per page accumulator: warp 1 the even page
+      // ordinals (U[0]), warp 3 the odd ones (U[1]).  Both release the S/P
+      // buffer, the V stage and the slot table of every tile.
+      const int par = warp == 1 ? 0 : 1;
       if (lane == 0) {
         uint32_t it = 0;
         bool ok = true;
@@ -1067,8 +1073,8 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
 #pragma unroll 1
             for (int q = 0; q < SLOTS && ok; ++q) {
               SlotMeta mt = sm.meta[s3][q];
-              if (mt.po < 0) continue;
-              int a = mt.po & 1;
+              if (mt.po < 0 || (mt.po & 1) != par) continue;
+              const int a = par;
               if ((mt.flags & 1) && mt.po >= 2) {
                 if (!mbar_wait(&sm.acc_empty[a], ((mt.po >> 1) - 1) & 1, kWait, abort_flag)) {
                   ok = false;
@@ -1086,8 +1092,8 @@ __device__ __forceinline__ void page_body(const TcLaunch &L, WsHeader *hdr, uint
           it += ntile;
         }
         if (*abort_flag) {
-          mma_commit(&sm.drain);  // every MMA issued by this thread has completed
-          mbar_wait_drain(&sm.drain, 0, kWait);
+          mma_commit(&sm.drain[par]);  // every MMA issued by this thread has completed
+          mbar_wait_drain(&sm.drain[par], 0, kWait);
         }
       }
     } else if (warp == 2) {
