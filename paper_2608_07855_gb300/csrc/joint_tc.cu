@@ -55,6 +55,7 @@ constexpr uint32_t kKHalf = kRound * kCT * 128;  // K rows of all pages, one hal
 constexpr uint32_t kVHalf = kCT * 128;           // V rows of one page, one half: 4 KB
 constexpr uint32_t kColS = 256;                  // TMEM column of page 0's S/P (kCT per page)
 constexpr int kHalfPad = 68;                     // floats per row of the o / D_A half buffers
+constexpr int kCached = 2;                       // groups per block whose row data stays in shared memory
 
 struct SmemJ {
   alignas(1024) uint8_t q[2 * kQHalf];
@@ -67,6 +68,11 @@ struct SmemJ {
   float Sc[kRound][kRows];     // S_E of every page and row (written by the page's team)
   int nc[kRound][kRows];       // n_E
   float part[kCombos + 1][kRows];  // team 1's sums of squares (and ||o||^2) for team 0
+  float part2[kCombos / 2 + 1][kRows];  // team 0's, for the subsets that team 1 evaluates
+  // the row data of the block's first kCached groups, kept from round to
+  // round: final max (base 2), exp-sum, visible count, position, S_A, n_A
+  float rc_m2[kCached][kRows], rc_l[kCached][kRows], rc_SA[kCached][kRows];
+  int rc_nvis[kCached][kRows], rc_qp[kCached][kRows], rc_nA[kCached][kRows];
   int pos[kRound][kCT];
   unsigned rmax[16];
   uint64_t bar;       // Q K^T done (one issuing thread)
@@ -446,13 +452,25 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
       const int hq = G.kvh * b.g + (rw.ok ? row / tr.W : 0), w = rw.ok ? row % tr.W : 0;
       rw.grow = L.row_off[G.t] + (int64_t)(G.li * b.H + G.kvh) * G.rows + (rw.ok ? row : 0);
       rw.st = L.stats[G.t] + (((int64_t)G.l * b.Hq + hq) * tr.W + w) * (D + 4);
-      const float mn = rw.ok ? rw.st[0] : -__builtin_huge_valf();
-      rw.m2 = mn == -__builtin_huge_valf() ? mn : mn * 1.4426950408889634f;
-      rw.l = rw.ok ? rw.st[1] : 0.0f;
-      rw.nvis = rw.ok ? (int)rw.st[2] : 0;
-      rw.qp = rw.ok ? tr.qpos[w] : -0x7fffffff;
-      rw.SA = rw.ok ? L.SA[rw.grow * 2] : 0.0f;
-      rw.nA = rw.ok ? (int)L.SA[rw.grow * 2 + 1] : 0;
+      // the block's k-th group; its row data is read from global memory in
+      // the first round and from the shared copy after that
+      const int kslot = (grp - (int)blockIdx.x) / (int)gridDim.x, rr = tid % kTeam;
+      if (kslot < kCached && r > 0) {
+        rw.m2 = s.rc_m2[kslot][rr];
+        rw.l = s.rc_l[kslot][rr];
+        rw.nvis = s.rc_nvis[kslot][rr];
+        rw.qp = s.rc_qp[kslot][rr];
+        rw.SA = s.rc_SA[kslot][rr];
+        rw.nA = s.rc_nA[kslot][rr];
+      } else {
+        const float mn = rw.ok ? rw.st[0] : -__builtin_huge_valf();
+        rw.m2 = mn == -__builtin_huge_valf() ? mn : mn * 1.4426950408889634f;
+        rw.l = rw.ok ? rw.st[1] : 0.0f;
+        rw.nvis = rw.ok ? (int)rw.st[2] : 0;
+        rw.qp = rw.ok ? tr.qpos[w] : -0x7fffffff;
+        rw.SA = rw.ok ? L.SA[rw.grow * 2] : 0.0f;
+        rw.nA = rw.ok ? (int)L.SA[rw.grow * 2 + 1] : 0;
+      }
       if (tid < 16) s.rmax[tid] = 0u;
 
       float2 ss2[kCombos], on2p = make_float2(0.0f, 0.0f);
@@ -477,31 +495,55 @@ __global__ void __launch_bounds__(kThreads, 1) joint_tc_kernel(const __grid_cons
           L.SA[rw.grow * 2 + 1] = (float)rw.nA;
         }
       }
+      if (kslot < kCached && tid < kTeam) {  // read again by both teams in the next round
+        s.rc_m2[kslot][rr] = rw.m2;
+        s.rc_l[kslot][rr] = rw.l;
+        s.rc_nvis[kslot][rr] = rw.nvis;
+        s.rc_qp[kslot][rr] = rw.qp;
+        s.rc_SA[kslot][rr] = rw.SA;
+        s.rc_nA[kslot][rr] = rw.nA;
+      }
       if (!run_pass<true>(s, L, hdr, G, rw, cand, kc, nf == 0, tm, lane_base, phase, phase_pv, ss2, on2p,
                           Sc, nc)) {
         ok = false;
         break;
       }
-      // the channel sums of the thread, then team 1's to team 0
+      // the channel sums of the thread; team 0 evaluates the subsets
+      // T = 1..8 and team 1 the subsets T = 9..15, each with the other team's
+      // sums of its channels added (one addition of two floats: the same
+      // value in either order)
+      constexpr int kSplit = kCombos / 2 + 1;  // subsets T <= kSplit go to team 0
       float ss[kCombos], on2 = on2p.x + on2p.y;
 #pragma unroll
       for (int i = 0; i < kCombos; ++i) ss[i] = ss2[i].x + ss2[i].y;
       if (tid >= kTeam) {
 #pragma unroll
-        for (int i = 0; i < kCombos; ++i) s.part[i][tid - kTeam] = ss[i];
-        s.part[kCombos][tid - kTeam] = on2;
+        for (int i = 0; i < kSplit; ++i) s.part[i][rr] = ss[i];
+        s.part[kCombos][rr] = on2;
+      } else {
+#pragma unroll
+        for (int i = kSplit; i < kCombos; ++i) s.part2[i - kSplit][rr] = ss[i];
+        s.part2[kCombos - kSplit][rr] = on2;
       }
       __syncthreads();
-      if (tid < kTeam) {
+      {
+        const int T0 = tid < kTeam ? 1 : kSplit + 1, T1 = tid < kTeam ? kSplit : kCombos;
+        if (tid < kTeam) {
 #pragma unroll
-        for (int i = 0; i < kCombos; ++i) ss[i] += s.part[i][tid];
-        on2 += s.part[kCombos][tid];
+          for (int i = 0; i < kSplit; ++i) ss[i] += s.part[i][rr];
+          on2 += s.part[kCombos][rr];
+        } else {
+#pragma unroll
+          for (int i = kSplit; i < kCombos; ++i) ss[i] += s.part2[i - kSplit][rr];
+          on2 += s.part2[kCombos - kSplit][rr];
+        }
         // Eq. 6 on A u T for every non-empty subset T of the round's pages;
         // S and n added in candidate order
         const float onorm = sqrtf(on2);
 #pragma unroll
         for (int T = 1; T < (1 << kRound); ++T) {
           if (T >= (1 << kc)) break;
+          if (T < T0 || T > T1) continue;
           float S_tot = rw.SA;
           int n_tot = rw.nA;
 #pragma unroll
