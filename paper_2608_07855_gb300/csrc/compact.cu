@@ -51,7 +51,7 @@ __device__ int block_scan(int v, int *excl, int *s_warp) {
   return total;
 }
 
-__global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant__ CompactLaunch L,
+__global__ void __launch_bounds__(kThreads, 1) select_kernel(const __grid_constant__ CompactLaunch L,
                                                           WsHeader *hdr) {
   int t = blockIdx.x;
   const TrajDev &tr = L.t[t];
@@ -181,17 +181,35 @@ __global__ void __launch_bounds__(kThreads) select_kernel(const __grid_constant_
         if ((key & mask) == prefix) atomicAdd(&s_hist[(key >> shift) & 255u], 1u);
       }
       __syncthreads();
-      if (threadIdx.x == 0) {
-        int need = s_krem;
-        unsigned cum = 0;
-        for (int d = 255; d >= 0; --d) {
-          if (cum + s_hist[d] >= (unsigned)need) {
-            s_prefix = prefix | ((unsigned long long)d << shift);
-            s_krem = need - (int)cum;
-            s_exact = s_krem == (int)s_hist[d];
-            break;
+      if (threadIdx.x < 32) {
+        // the first bin, from the top, at which the count of larger keys
+        // reaches `need`: lane l holds bins 255 - 8 l down to 248 - 8 l, a
+        // warp scan gives each lane the count above its bins, and the lane
+        // whose bins hold the crossing walks them in order
+        const int lane = threadIdx.x, need = s_krem;
+        unsigned sum = 0;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) sum += s_hist[255 - 8 * lane - u];
+        unsigned incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const unsigned hit = __ballot_sync(0xffffffffu, incl >= (unsigned)need);
+        if (hit != 0u && lane == __ffs(hit) - 1) {
+          unsigned cum = incl - sum;
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const unsigned c = s_hist[255 - 8 * lane - u];
+            if (cum + c >= (unsigned)need) {
+              s_prefix = prefix | ((unsigned long long)(255 - 8 * lane - u) << shift);
+              s_krem = need - (int)cum;
+              s_exact = s_krem == (int)c;
+              break;
+            }
+            cum += c;
           }
-          cum += s_hist[d];
         }
       }
       mask |= 255ull << shift;

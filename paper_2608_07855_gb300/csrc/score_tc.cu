@@ -157,8 +157,8 @@ __device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int 
 // output accumulator, so one warpgroup's softmax overlaps the other's MMAs.
 // TMEM columns: S/P buffer b at 128 b (after the softmax reads a 32-column
 // chunk of S it overwrites the same columns with 16 columns of P_hi and 16
-// of P_lo), O_b at 256 + 128 b.  Each item writes two partials, one per
-// warpgroup.
+// of P_lo), O_b at 256 + 128 b.  At the end of an item the two warpgroups
+// merge their states in the CTA and write one partial.
 struct SmemA {
   alignas(1024) uint8_t q[kTileBytes];
   alignas(1024) uint8_t k[NKB][kTileBytes];
@@ -669,6 +669,12 @@ __device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int 
   // headers, one partial per lane: (reference max, sum, visible count, true max)
   const float4 h0 = lane < nparts ? ld_once(part(lane)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
   const float4 h1 = lane + 32 < nparts ? ld_once(part(lane + 32)) : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+  // the first kBatch partials' outputs, four channels per lane, loaded
+  // before the weights are known (the loads depend on nothing)
+  constexpr int kBatch = FUSED ? 2 : 8;  // the fused launch's merge warps run on 48 registers
+  float4 vb[kBatch];
+#pragma unroll
+  for (int u = 0; u < kBatch; ++u) vb[u] = u < nparts ? ld_once(part(u) + 4 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
   const float m = warp_max(fmaxf(h0.w, h1.w));  // true row max over the partials (base 2)
   // weight of each partial; a partial that saw nothing (reference -inf) has
   // weight 0 and an unwritten output
@@ -677,17 +683,26 @@ __device__ __forceinline__ void merge_row(const TcLaunch &L, int t, int li, int 
   const float lsum = warp_sum(fmaf(h0.y, a0, h1.y * a1));
   const float n = warp_sum(h0.z + h1.z);
   float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-  // outputs, four channels per lane, partials in order; the loads do not
-  // depend on each other
-#pragma unroll 8
-  for (int k = 0; k < nparts; ++k) {
-    const float a = __shfl_sync(0xffffffffu, k < 32 ? a0 : a1, k & 31);
-    float4 v = ld_once(part(k) + 4 + lane * 4);
-    if (a == 0.0f) v = make_float4(0.f, 0.f, 0.f, 0.f);
-    o.x = fmaf(v.x, a, o.x);
-    o.y = fmaf(v.y, a, o.y);
-    o.z = fmaf(v.z, a, o.z);
-    o.w = fmaf(v.w, a, o.w);
+  // outputs, partials in order, in batches whose loads are issued
+  // together
+  for (int k0 = 0; k0 < nparts; k0 += kBatch) {
+    if (k0 > 0) {
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u)
+        vb[u] = k0 + u < nparts ? ld_once(part(k0 + u) + 4 + lane * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int k = k0 + u;
+      const float a = __shfl_sync(0xffffffffu, k < 32 ? a0 : a1, k & 31);
+      if (k >= nparts) break;
+      float4 v = vb[u];
+      if (a == 0.0f) v = make_float4(0.f, 0.f, 0.f, 0.f);
+      o.x = fmaf(v.x, a, o.x);
+      o.y = fmaf(v.y, a, o.y);
+      o.z = fmaf(v.z, a, o.z);
+      o.w = fmaf(v.w, a, o.w);
+    }
   }
   const float inv = lsum > 0.0f ? 1.0f / lsum : 0.0f;
   const int h = kvh * L.g + row / tr.W, w = row % tr.W;
