@@ -211,3 +211,44 @@ def test_oracle_decode_checkpoint_keeps_the_most_attended_tokens():
     kept[I] = True
     f32 = fill.astype(np.float32)
     assert f32[kept].min() >= f32[~kept].max()
+
+
+def test_decode_checkpoint_after_a_commit_protects_nothing():
+    """Once a commit's post-commit decisions are taken no page awaits its
+    measurement, so a decode checkpoint has no pending set to protect (Eq. 12's
+    N_j is empty) even with a protection cap: among the tokens that are not
+    retired, the budget goes to the highest fill scores alone."""
+    cfg = synth.small_config("timeline", event_len=(24, 80), G=16, M=1, H=1, Hq=4)
+    tl = synth.make_timeline(cfg, 4, 3)
+    K64, V64 = synth.values_f64(tl.K, cfg.dtype), synth.values_f64(tl.V, cfg.dtype)
+    B = 160
+    o = OracleSession(cfg.M, cfg.H, cfg.Hq, cfg.d, cfg.G, B, 0.25, protect_cap=4, thresholds=TH, tau_joint=0.6)
+    end, posted = 0, False
+    for step in synth.timeline_steps(tl):
+        if step[0] == "append":
+            a, b = step[1], step[2]
+            o.append(K64[:, :, a:b], V64[:, :, a:b], np.arange(a, b), synth.timeline_events(tl, a, b))
+            end = b
+            if posted:
+                break  # the tokens decoded after the first commit's decisions
+        elif step[0] == "pre":
+            o.pre_commit(synth.values_f64(tl.Q_pre[step[1]], cfg.dtype), tl.qpos_pre(step[1]))
+        elif step[0] == "post":
+            o.post_commit(synth.values_f64(tl.Q_post[step[1]], cfg.dtype), tl.qpos_post(step[1]))
+            posted = True
+    assert posted and o.measured == []
+    q, qp = tl.window(end)
+    q64 = synth.values_f64(q, cfg.dtype)
+    fill = o.fill_scores(q64, qp).astype(np.float32)
+    retired_tok = np.zeros(o.pos.shape[0], bool)
+    for pid, s, n in o.pages:
+        if pid in o.retired:
+            retired_tok[s:s + n] = True
+    live = ~retired_tok
+    assert live.sum() > B
+    I = o.decode_checkpoint(q64, qp)
+    assert len(I) == B
+    kept = np.zeros(fill.shape[0], bool)
+    kept[I] = True
+    assert not kept[retired_tok].any()
+    assert fill[kept & live].min() >= fill[~kept & live].max()

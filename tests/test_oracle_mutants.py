@@ -66,7 +66,7 @@ def _failing(checks):
     for name, fn in checks:
         try:
             fn()
-        except (AssertionError, ValueError):
+        except Exception:  # an assertion, or the mistake made the pin's own run fail
             failed.append(name)
     return failed
 
@@ -153,3 +153,61 @@ def test_pins_reject_python_mutant(fn, what, old, new, monkeypatch):
     monkeypatch.setattr(core, fn, ns[fn])
     failed = _failing(_selection_pins())
     assert failed, f"no pin rejects the mistake: {fn}: {what}"
+
+
+# ----------------------------------------------------------------------------
+# the multi-commit driver (Algorithm 1's outer loop)
+
+import textwrap  # noqa: E402
+
+import test_oracle_lifecycle as lpins  # noqa: E402
+from oracle import lifecycle  # noqa: E402
+
+
+def _lifecycle_pins():
+    return [
+        ("hand-worked timeline", lpins.test_hand_worked_timeline),
+        ("hand-worked timeline, scan cap 0", lpins.test_hand_worked_timeline_scan_cap),
+        ("timeline invariants", lpins.test_oracle_lifecycle_invariants),
+        ("decode checkpoint after a commit", lpins.test_decode_checkpoint_after_a_commit_protects_nothing),
+    ]
+
+
+# (method of OracleSession, what the mistake is, the text it replaces, the mistaken text)
+LIFECYCLE_MUTANTS = [
+    ("post_commit", "every non-retired resident page is in E_c, the new observation's included",
+     "eligible = np.asarray([pid in meas and pid not in self.retired for pid in ids], np.uint8)",
+     "eligible = np.asarray([pid not in self.retired for pid in ids], np.uint8)"),
+    ("post_commit", "the candidate list is not cut to the scan cap",
+     "cand = cand[:self.scan_cap]", "cand = cand"),
+    ("post_commit", "accepted pages do not join D_c",
+     "self.retired |= set(accepted)", "pass"),
+    ("pre_commit", "retired pages are measured again",
+     "self.measured = [pid for pid in self.page_ids() if pid not in self.retired]",
+     "self.measured = list(self.page_ids())"),
+    ("checkpoint_resident", "a partly retained page keeps its old first row",
+     "pages.append([pid, int(new_index[s + kept[0]]), len(kept)])",
+     "pages.append([pid, int(new_index[s]), len(kept)])"),
+    ("checkpoint_resident", "a partly retained page keeps its old length",
+     "pages.append([pid, int(new_index[s + kept[0]]), len(kept)])",
+     "pages.append([pid, int(new_index[s + kept[0]]), n])"),
+    ("checkpoint_resident", "every non-retired page is protected as pending",
+     "pend = [i for i, pid in enumerate(ids) if pid in set(self.measured)]",
+     "pend = [i for i, pid in enumerate(ids) if pid not in self.retired]"),
+]
+
+
+@pytest.mark.parametrize("meth,what,old,new", LIFECYCLE_MUTANTS,
+                         ids=[f"{m[0]}: {m[1]}" for m in LIFECYCLE_MUTANTS])
+def test_pins_reject_lifecycle_mutant(meth, what, old, new, monkeypatch):
+    src = textwrap.dedent(inspect.getsource(getattr(lifecycle.OracleSession, meth)))
+    assert src.count(old) == 1, what
+    ns = dict(lifecycle.__dict__)
+    exec(compile(src.replace(old, new), f"<mutant of OracleSession.{meth}>", "exec"), ns)
+    monkeypatch.setattr(lifecycle.OracleSession, meth, ns[meth])
+    failed = _failing(_lifecycle_pins())
+    assert failed, f"no pin rejects the mistake: {meth}: {what}"
+
+
+def test_lifecycle_pins_accept_the_oracle():
+    assert _failing(_lifecycle_pins()) == []
