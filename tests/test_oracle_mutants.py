@@ -53,6 +53,9 @@ def _effect_pins():
 
 def _selection_pins():
     return [
+        ("token scores, uniform attention", pins.test_token_scores_uniform_attention),
+        ("token scores, invariants", pins.test_token_scores_invariants),
+        ("token scores, C row statistics", pins.test_token_scores_match_row_stats),
         ("classify hand table", lambda: pins.test_classify_hand(GOLDEN)),
         ("classify ablations hand table", lambda: pins.test_classify_variants_hand(GOLDEN)),
         *[(f"classify properties, seed {s}", (lambda s=s: pins.test_classify_properties(s))) for s in range(5)],
@@ -90,6 +93,16 @@ C_MUTANTS = [
      "s[i] = vis[i] ? pb->scale * dot(", "s[i] = vis[i] ? dot("),
     ("deleting every visible token gives 0 instead of rule (2)",
      "r = OKV_INF; /* rule (2) */", "r = 0.0; /* rule (2) */"),
+    ("the greedy scan (explicit deletion) accepts only below tau",
+     "    step_R[j] = R;\n    if (R <= tau) {\n      accepted[E] = 1;\n      memcpy(drop, trial, pb->S);",
+     "    step_R[j] = R;\n    if (R < tau) {\n      accepted[E] = 1;\n      memcpy(drop, trial, pb->S);"),
+    ("the greedy scan (closed form) accepts only below tau",
+     "    step_R[j] = R;\n    if (R <= tau) {\n      accepted[E] = 1;\n      greedy_pass(&base, rows, nthreads, E, 1);",
+     "    step_R[j] = R;\n    if (R < tau) {\n      accepted[E] = 1;\n      greedy_pass(&base, rows, nthreads, E, 1);"),
+    ("the greedy scan (explicit deletion) forgets accepted pages",
+     "      accepted[E] = 1;\n      memcpy(drop, trial, pb->S);", "      accepted[E] = 1;"),
+    ("the greedy scan (closed form) does not fold accepted pages into D",
+     "      accepted[E] = 1;\n      greedy_pass(&base, rows, nthreads, E, 1);", "      accepted[E] = 1;"),
 ]
 
 
@@ -141,6 +154,14 @@ PY_MUTANTS = [
      "key=lambda i: (-float(fill_score[i]), -i)", "key=lambda i: (float(fill_score[i]), -i)"),
     ("select_indices", "retired pages not excluded",
      "tok_retired[page_start[E]: page_start[E] + page_len[E]] = True", "pass"),
+    ("token_scores", "a token's weights summed over the rows instead of maximised",
+     "score[idx] = np.maximum(score[idx], e / e.sum())", "score[idx] = score[idx] + e / e.sum()"),
+    ("token_scores", "the weights not normalised by the row's sum",
+     "score[idx] = np.maximum(score[idx], e / e.sum())", "score[idx] = np.maximum(score[idx], e)"),
+    ("token_scores", "the causal mask drops the query's own position",
+     "vis = pb.pos <= pb.qpos[w]", "vis = pb.pos < pb.qpos[w]"),
+    ("token_scores", "a query head reads the wrong KV head",
+     "Kh = pb.K[li, h // g]", "Kh = pb.K[li, h % pb.H]"),
 ]
 
 
