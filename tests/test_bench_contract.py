@@ -82,3 +82,15 @@ def test_joint_report_counts():
     r = bench.joint_report(buf, 0.7)
     assert r["n_cand"] == 7 and r["accepted"] == 4 and r["rejected"] == 3
     assert r["rounds"] == 2 and abs(r["us_per_candidate"] - 100.0) < 1e-9
+
+
+def test_recorded_traffic_belongs_to_the_current_kernels():
+    """The DRAM bytes bench.py reports as roofline.traffic were captured with
+    the scoring sources as they are now (their sha256 prefix), and lie
+    between once and three times the algorithmic bytes of the step."""
+    cfg = synth.CONFIGS["qwen3_8b_32k"]
+    traffic, sha = bench.MEASURED_TRAFFIC[cfg.name]
+    assert sha == bench.scoring_sources_sha()
+    bpt, _ = bench.algorithmic(cfg)
+    algo = bpt * (32768 + (32768 + 4096 + 32))
+    assert algo <= traffic <= 3 * algo
